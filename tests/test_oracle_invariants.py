@@ -1,0 +1,146 @@
+"""Scheduler invariants of the oracle, re-derived from its per-call logs.
+
+For each call the release time is rebuilt from the workflow of Sec. 2.1
+(S at arrival; G_c after S; C_{c,r} after its predecessor in chain c; E after
+the last call of every chain) and checked against the log:
+  - dispatch happens at release and no call starts before it is released;
+  - an instance never runs more calls than it has slots;
+  - work conservation: while a call waits, its instance has no free slot;
+  - each call runs exactly once for its service time;
+  - P95, SLO count, makespan and the digest agree with the logged times.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2505_05286_gb300 import workloads as W
+
+
+def _release_times(tr, end):
+    rel = np.full(tr.n_calls, -1, np.int64)
+    for i in range(tr.n_queries):
+        b, e = int(tr.call_base[i]), int(tr.call_base[i + 1])
+        rel[b] = tr.arrival_us[i]
+        last_of_chain = {}
+        for j in range(b + 1, e - 1):
+            c = int(tr.cand[j])
+            if tr.stage[j] == W.STAGE_G:
+                rel[j] = end[b]
+            else:
+                rel[j] = end[last_of_chain[c]]
+            last_of_chain[c] = j
+        rel[e - 1] = max(end[j] for j in last_of_chain.values())
+    return rel
+
+
+def _mix64(z):
+    m = (1 << 64) - 1
+    z &= m
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & m
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & m
+    return z ^ (z >> 31)
+
+
+def check_schedule(tr, cl, res, log):
+    p = oracle.prep(tr, cl)
+    inst, enq, start, end = log["inst"], log["enq"], log["start"], log["end"]
+    assert (inst >= 0).all() and (start >= 0).all()
+    rel = _release_times(tr, end)
+    assert (enq == rel).all(), "dispatch must happen when the predecessors finish"
+    assert (start >= enq).all()
+    types = cl.inst_type[inst]
+    assert (end - start == p["svc"][np.arange(tr.n_calls), types]).all()
+    for m in range(cl.n_inst):
+        slots = int(cl.slots[cl.inst_type[m]])
+        on = np.nonzero(inst == m)[0]
+        if on.size == 0:
+            continue
+        times = np.unique(np.concatenate([start[on], end[on], enq[on]]))
+        # running count after all events at time t
+        running = np.array([np.sum((start[on] <= t) & (end[on] > t)) for t in times])
+        assert running.max() <= slots
+        for c in on[start[on] > enq[on]]:
+            sel = (times >= enq[c]) & (times < start[c])
+            assert (running[sel] == slots).all(), "a call waited while a slot was free"
+    lat = end[tr.call_base[1:] - 1] - tr.arrival_us
+    n = tr.n_queries
+    assert int(res["n_done"]) == n and int(res["events"]) == tr.n_calls
+    if n:
+        rank = -(-95 * n // 100)
+        assert int(res["p95_us"]) == int(np.sort(lat)[rank - 1])
+        assert int(res["slo_met"]) == int(np.sum(lat <= p["t_slo"]))
+        assert int(res["makespan_us"]) == int(end.max())
+    dig = 0
+    for c in range(tr.n_calls):
+        dig += _mix64(int(start[c]) ^ _mix64((c << 8) | int(inst[c])))
+    for i in range(n):
+        dig += _mix64(int(end[tr.call_base[i + 1] - 1]) ^ _mix64((i << 8) | 0xFF))
+    assert dig % (1 << 64) == int(res["digest"])
+
+
+CASES = [
+    (0, None, None, list(range(16))),
+    (1, 1, 250, [0, 7, 9, 36, 63]),
+    (2, 1, 200, [0, 5, 77, 130, 255]),
+    (3, 1, 200, [0, 100, 300, 511]),
+    (4, 1, 150, [0, 517, 1023]),
+]
+
+
+@pytest.mark.parametrize("cfg,nt,nq,points", CASES)
+def test_invariants_pq_wb(cfg, nt, nq, points):
+    wl = W.make_workload(cfg, n_traces=nt, n_queries=nq)
+    tr = wl.traces[0]
+    for p in points:
+        res, log = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, p), check=True, log=True)
+        assert res["status"] == 0
+        check_schedule(tr, wl.cluster, res, log)
+
+
+@pytest.mark.parametrize("local,dispatch", [(W.POLICY_FCFS, W.DISPATCH_WB), (W.POLICY_PQ, W.DISPATCH_RR),
+                                            (W.POLICY_FCFS, W.DISPATCH_RR)])
+def test_invariants_policies(local, dispatch):
+    wl = W.make_workload(1, n_traces=1, n_queries=200)
+    tr = wl.traces[0]
+    for p in [0, 18, 63]:
+        pt = oracle.point_of(wl.grid, p)
+        pt["local_policy"], pt["dispatch_policy"] = local, dispatch
+        res, log = oracle.simulate(tr, wl.cluster, pt, check=True, log=True)
+        assert res["status"] == 0
+        check_schedule(tr, wl.cluster, res, log)
+
+
+def test_overloaded_queue():
+    """alpha = 1 sends everything to the fastest instance: a long queue forms
+    and the invariants still hold."""
+    wl = W.make_workload(4, n_traces=1, n_queries=400)
+    tr = wl.traces[0]
+    pt = oracle.point_of(wl.grid, wl.grid.n_points - 1)
+    res, log = oracle.simulate(tr, wl.cluster, pt, check=True, log=True)
+    assert res["status"] == 0
+    check_schedule(tr, wl.cluster, res, log)
+    assert len(set(log["inst"].tolist())) == 1
+    waits = log["start"] - log["enq"]
+    assert waits.max() > 2 * 10 ** 6  # queued for more than 2 s
+
+
+def test_empty_trace():
+    wl = W.make_workload(0, n_queries=0)
+    res = oracle.simulate(wl.traces[0], wl.cluster, oracle.point_of(wl.grid, 0), check=True)
+    assert res["status"] == 0 and res["n_done"] == 0 and res["p95_us"] == 0 and res["digest"] == 0
+
+
+def test_rejects_malformed():
+    wl = W.make_workload(0, n_queries=5)
+    tr = wl.traces[0]
+    bad = W.Trace(*[getattr(tr, f).copy() for f in ("arrival_us", "k", "call_base", "prompt", "out",
+                                                       "out_est", "stage", "cand", "retry")])
+    bad.arrival_us[2] = bad.arrival_us[1] - 1  # unsorted
+    assert oracle.simulate(bad, wl.cluster, oracle.point_of(wl.grid, 0))["status"] == 1
+    bad2 = W.Trace(*[getattr(tr, f).copy() for f in ("arrival_us", "k", "call_base", "prompt", "out",
+                                                        "out_est", "stage", "cand", "retry")])
+    bad2.stage[1] = W.STAGE_E  # broken workflow structure
+    assert oracle.simulate(bad2, wl.cluster, oracle.point_of(wl.grid, 0))["status"] == 1
+    pt = oracle.point_of(wl.grid, 0)
+    pt["alpha_fp"] = W.SCALE + 1
+    assert oracle.simulate(tr, wl.cluster, pt)["status"] == 1
