@@ -1,0 +1,305 @@
+"""Benchmark of the batched HexGen-Flow scheduler simulation on GB300.
+
+One step = one pass of the whole path through the C ABI (`hx_sim_run`):
+per-call preparation, every (trace x point) simulation, the best-point
+reduction, on the ceiling workload (256 traces x 20000 queries, 64
+instances of 4 types, 1024 hyper-parameter points = 262144 simulations).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints one JSON line.  `value` is simulations per second over the timed
+steps (inputs resident in HBM; they are larger than L2, so no flush is
+needed).  `e2e` is the same metric through the C ABI from host buffers:
+upload of the traces, the run, and the read-back of the results per step.
+`--impl reference` times the CPU oracle (plain C, one simulation per
+process, all host cores) on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2505_05286_gb300 import workloads as W  # noqa: E402
+
+CFG = 4
+METRIC = "scheduler sims/sec (hyperparam×trace) and simulated stage-events/sec on 1 GB300"
+UNIT = "sims/s"
+L2_BYTES = 129 * 2 ** 20
+SM_COUNT_FALLBACK = 152
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples during the timed region."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 8:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def _barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def _max_over_ranks(world, x: float) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def oracle_sample(wl, n_sims: int, seed: int, procs: int):
+    """Seeded sample of simulations of `wl` run by the CPU oracle."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    sims = sorted(rng.choice(wl.n_sims, size=min(n_sims, wl.n_sims), replace=False).tolist())
+    t0 = time.perf_counter()
+    oracle.run(wl, sims, procs=procs)
+    dt = time.perf_counter() - t0
+    P = wl.grid.n_points
+    events = sum(wl.traces[s // P].n_calls for s in sims)
+    return len(sims), events, dt, sims
+
+
+def cpu_baseline(wl, budget_s: float = 20.0):
+    procs = os.cpu_count() or 1
+    n, events, dt, _ = oracle_sample(wl, max(procs, 16), 7, procs)
+    # scale the sample toward the time budget once
+    if dt < budget_s / 3:
+        extra = int(n * (budget_s / max(dt, 1e-3) - 1))
+        extra = max(0, min(extra, 4 * procs * 4))
+        if extra:
+            n2, e2, dt2, _ = oracle_sample(wl, extra, 8, procs)
+            n, events, dt = n + n2, events + e2, dt + dt2
+    return {"value": n / dt, "unit": UNIT, "cores": procs, "kind": "oracle",
+            "events_per_s": events / dt,
+            "sample": f"{n} seeded random simulations of {wl.name}, one per process, {procs} processes, "
+                      f"{dt:.1f} s wall"}
+
+
+def run_reference(args):
+    world, rank, _ = _dist()
+    if rank != 0:
+        return
+    wl = W.make_workload(CFG)
+    procs = os.cpu_count() or 1
+    per_step = max(procs, 16)
+    for w in range(args.warmup):
+        oracle_sample(wl, max(2, procs // 4), 1000 + w, procs)
+    t = 0.0
+    n_tot = ev_tot = 0
+    for k in range(args.steps):
+        n, ev, dt, _ = oracle_sample(wl, per_step, 2000 + k, procs)
+        t += dt
+        n_tot += n
+        ev_tot += ev
+    value = n_tot / t
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * t / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+            "data": "synthetic", "stage_events_per_s": ev_tot / t,
+            "config": {"workload": wl.name, "sims": wl.n_sims, "sample_sims_per_step": per_step,
+                       "l2": "oracle on host cores"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": procs, "kind": "oracle",
+                             "sample": f"{per_step} seeded random simulations per step, one per process"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_gpu(args):
+    import torch
+    world, rank, local = _dist()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    from paper_2505_05286_gb300 import build as B
+    from paper_2505_05286_gb300 import hxsim as H
+    B.build()
+    # weak scaling: every rank simulates its own 256 traces (trace seeds offset by rank)
+    wl = W.make_workload(CFG, first_trace=rank * W.CONFIGS[CFG].n_traces)
+    n_calls = wl.n_calls
+    P = wl.grid.n_points
+    sim = H.Sim(wl.traces, wl.cluster, wl.grid, timing=True)
+    info = sim.info()
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        sim.run(stream)
+    torch.cuda.synchronize()
+
+    # kernel-only timing: inputs resident, K steps between events on the stream
+    sim_ms = []
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    _barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for _ in range(args.steps):
+            sim.run(stream)
+        stop.record(stream)
+        torch.cuda.synchronize()
+    _barrier(world)
+    t_ms = start.elapsed_time(stop)
+    # per-kernel times of the last timed step (events the library records on the same stream)
+    sim_ms.append(sim.timings())
+    t_ms = _max_over_ranks(world, t_ms)
+    res = sim.results()
+    ok = bool((res["status"] == 0).all())
+    events_per_step = int(res["events"].sum())
+    sims_total = wl.n_sims * world
+    value = sims_total * args.steps / (t_ms / 1000.0)
+    events_rate = events_per_step * world * args.steps / (t_ms / 1000.0)
+    prep_ms = float(np.median([x[0] for x in sim_ms]))
+    kern_ms = float(np.median([x[1] for x in sim_ms]))
+    best_ms = float(np.median([x[2] for x in sim_ms]))
+
+    # end to end through the C ABI from host buffers: upload, run, read back
+    e2e_steps = max(1, min(args.steps, 3))
+    h2d = sum(t.arrival_us.nbytes + t.k.nbytes + t.call_base.nbytes + t.prompt.nbytes + t.out.nbytes +
+              t.out_est.nbytes + t.stage.nbytes + t.cand.nbytes + t.retry.nbytes for t in wl.traces)
+    d2h = wl.n_sims * H.RESULT_DTYPE.itemsize
+    _barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        sim.upload(wl.traces, stream)
+        sim.run(stream)
+        res2 = sim.results()
+    torch.cuda.synchronize()
+    e2e_s = _max_over_ranks(world, time.perf_counter() - t0)
+    ok = ok and bool((res2["digest"] == res["digest"]).all())
+    e2e_value = sims_total * e2e_steps / e2e_s
+    best = sim.best(wl.objective)
+
+    peaks, peak_kind = _peaks()
+    clocks = clk.summary()
+    # roofline of the dominant kernel (the simulation kernel): SM issue slots
+    sm_count = torch.cuda.get_device_properties(0).multi_processor_count
+    sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
+    peak_warp_inst = sm_count * 4 * sm_mhz * 1e6          # warp instructions per second
+    n_inst = wl.cluster.n_inst
+    alg_per_event = 6 * n_inst + 40                         # int ops per call event (algorithmic)
+    lane_peak = sm_count * 128 * sm_mhz * 1e6               # 32-bit lane operations per second
+    achieved = alg_per_event * events_per_step / (kern_ms / 1000.0)
+    roofline = {"bound": "alu", "achieved": achieved / 1e9, "peak": lane_peak / 1e9, "unit": "Gop/s",
+                "frac": achieved / lane_peak, "traffic": None,
+                "ops_per_event": alg_per_event, "events_per_launch": events_per_step,
+                "kernel": "hx_sim_kernel", "kernel_ms": kern_ms,
+                "peak_source": f"{sm_count} SMs x 128 int32 lanes x {sm_mhz:.0f} MHz ({peak_kind} sm_max_mhz)",
+                "issue_peak_ginst_s": peak_warp_inst / 1e9}
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "stage_events_per_s": events_rate, "all_sims_ok": ok,
+            "config": {"workload": wl.name, "traces": len(wl.traces), "queries_per_trace": W.CONFIGS[CFG].n_queries,
+                       "instances": n_inst, "points": P, "sims": wl.n_sims, "calls": n_calls,
+                       "l2": f"inputs larger than L2 ({n_calls * 64 / 2**30:.2f} GiB of call records)",
+                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                       "resident_warps": info["resident_warps"], "blocks": info["blocks"]},
+            "kernels_ms": {"prep": prep_ms, "simulate": kern_ms, "best": best_ms},
+            "best_point": {"global_point": best[0], "sum_p95_us": best[1], "sum_slo_met": best[2]},
+            "roofline": roofline, "clocks": clocks, "gpu_launches": 3 * args.steps,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+                    "steps": e2e_steps}}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    sim.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

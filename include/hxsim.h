@@ -1,0 +1,217 @@
+/*
+ * hxsim.h -- C ABI of the batched HexGen-Flow scheduler simulation on GB300.
+ *
+ * HexGen-Flow (arXiv 2505.05286) tunes its dispatcher weight alpha by
+ * replaying a recent request trace through a simulator of its own two-level
+ * scheduler and keeping the point with the lowest simulated P95 latency
+ * (Sec. 4.3, Eq. alpha* = argmin T_0.95(alpha)).  This library runs that
+ * simulation for many (hyper-parameter point x trace) pairs at once on one
+ * GPU: one warp simulates one pair, event by event, and a final kernel picks
+ * the best point.
+ *
+ * What one simulation computes (all times int64 microseconds; alpha, gamma
+ * and the SLO multiplier fixed point with HX_SCALE = 1e6; every division
+ * truncates toward zero):
+ *  - the workflow of Sec. 2.1 / Sec. 3.3: a query issues schema linking (S),
+ *    then k candidate generations (G_c) in parallel, each followed by its
+ *    self-correction calls C_{c,1..r_c}, then evaluation (E) once every
+ *    chain has finished; a call is dispatched the moment it is released;
+ *  - Eq. (comp): t_comp = ceil(prompt * 1e6 / prefill_tok_s)
+ *    + out_est * decode_us_tok on the instance's type (true `out` gives the
+ *    service time);
+ *  - the dispatch score of Eq. (score), in fixed point:
+ *    S_m = (SCALE - A) * min(beta / max(t_queue_m, 1), 2^43 - 1) - A * t_comp_m,
+ *    t_queue_m = sum of t_comp over the requests dispatched to m and not yet
+ *    finished; the highest score wins, ties to the lowest instance index;
+ *  - the SLO budget of Sec. 4.2 at dispatch:
+ *    t_slo = (T_slo - elapsed) * tbar / (tbar + rest of this request's path),
+ *    tbar = mean of t_comp over instances, the rest = stage reference costs
+ *    of G, min(rho, R - u) corrections and E as applicable;
+ *  - Eq. (priority) with ageing weight gamma: U = t_comp - t_slo + gamma*tau;
+ *    at each batch boundary an instance starts its highest-U waiting request
+ *    (ties to the lowest request id);
+ *  - events in the order (time, completions before arrivals, instance,
+ *    request id / query id);
+ *  - per simulation the nearest-rank P95 of query latencies
+ *    (sorted L[ceil(0.95 n) - 1]), the number of queries with latency <= T_slo,
+ *    T_slo = slo_mult * (S + slowest chain + E on the reference type).
+ *
+ * Errors: every function returns an HX_* status; nothing throws or aborts
+ * across the ABI.  hx_last_error() returns the calling thread's last message.
+ * Ownership: the caller keeps its host buffers (they may be freed once
+ * hx_sim_create returns); the library owns all device memory of a handle.
+ */
+#ifndef HXSIM_H
+#define HXSIM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define HX_SCALE 1000000LL
+
+enum {
+  HX_OK = 0,
+  HX_ERR_INVALID = 1,    /* malformed or out-of-range input */
+  HX_ERR_CUDA = 2,       /* a CUDA runtime call failed */
+  HX_ERR_OOM = 3,        /* device or host allocation failed */
+  HX_ERR_CAPACITY = 4,   /* a simulation outgrew its scratch (per-sim status) */
+  HX_ERR_STEP_LIMIT = 5, /* a simulation exceeded its event bound (per-sim status) */
+  HX_ERR_STATE = 6       /* call out of order (e.g. results before run) */
+};
+
+enum { HX_STAGE_S = 0, HX_STAGE_G = 1, HX_STAGE_C = 2, HX_STAGE_E = 3 };
+enum { HX_LOCAL_PQ = 0, HX_LOCAL_FCFS = 1 };
+enum { HX_DISPATCH_WB = 0, HX_DISPATCH_RR = 1 };
+enum { HX_OBJ_P95 = 0, HX_OBJ_P95_SLO95 = 1 };
+
+/* Limits checked by hx_sim_create. */
+#define HX_MAX_INST 64
+#define HX_MAX_TYPES 4
+#define HX_MAX_SLOTS 16
+#define HX_MAX_K 8
+#define HX_MAX_RETRY 15
+
+/* One request trace (host memory).  Calls of query i are
+ * [call_base[i], call_base[i+1]) in the order S, G_0..G_{k-1}, the
+ * corrections C_{c,r} by (c, r) ascending (r = 1..r_c), then E.
+ * The request id of a call is its index within the trace. */
+typedef struct hx_trace {
+  int32_t n_queries;
+  int32_t n_calls;              /* < 2^24 */
+  const int64_t* arrival_us;    /* [n_queries] non-decreasing, >= 0 */
+  const uint8_t* k;             /* [n_queries] 1..8 */
+  const int32_t* call_base;     /* [n_queries + 1] */
+  const int32_t* prompt;        /* [n_calls] >= 1 */
+  const int32_t* out;           /* [n_calls] true output tokens >= 0 */
+  const int32_t* out_est;       /* [n_calls] scheduler's believed output tokens >= 0 */
+  const uint8_t* stage;         /* [n_calls] HX_STAGE_* */
+  const uint8_t* cand;          /* [n_calls] candidate c (G and C calls) */
+  const uint8_t* retry;         /* [n_calls] r for C calls, 0 otherwise */
+} hx_trace;
+
+/* Heterogeneous instances (Sec. 3.3's empirical performance profiles). */
+typedef struct hx_cluster {
+  int32_t n_types;                  /* 1..4 */
+  const int32_t* prefill_tok_s;     /* [n_types] >= 1 */
+  const int32_t* decode_us_tok;     /* [n_types] >= 0 */
+  const int32_t* slots;             /* [n_types] 1..16 concurrent requests */
+  int32_t n_inst;                   /* 1..64 */
+  const uint8_t* inst_type;         /* [n_inst] */
+  int32_t ref_type;                 /* type whose exclusive latency defines T_slo */
+  int64_t slo_mult_fp;              /* T_slo = slo_mult_fp * L0 / SCALE, <= 16 * SCALE */
+  int32_t rmax;                     /* workflow's retry bound R, 0..15 */
+  const int32_t* stage_ref_prompt;  /* [4] reference tokens per stage (S,G,C,E) */
+  const int32_t* stage_ref_out;     /* [4] */
+} hx_cluster;
+
+/* Hyper-parameter points (host memory). */
+typedef struct hx_grid {
+  int32_t n_points;
+  const int64_t* alpha_fp;          /* [n] 0..SCALE (Eq. score's alpha) */
+  const int64_t* gamma_fp;          /* [n] 0..4*SCALE (urgency ageing weight) */
+  const int32_t* rho;               /* [n] 0..15 corrections assumed by the budget */
+  const int64_t* beta_us2;          /* [n] >= 0, beta = C_ref * Q_ref */
+  const uint8_t* local_policy;      /* [n] HX_LOCAL_* */
+  const uint8_t* dispatch_policy;   /* [n] HX_DISPATCH_* */
+} hx_grid;
+
+typedef struct hx_options {
+  int32_t n_record;                 /* simulations whose per-call log is kept */
+  const int32_t* record_sims;       /* [n_record] sim indices (trace * P + point) */
+  int32_t max_resident_warps;       /* 0 = fill the GPU */
+  int32_t timing;                   /* 1 = time each kernel with CUDA events */
+} hx_options;
+
+/* Per-simulation result, index sim = trace * n_points + point. */
+typedef struct hx_result {
+  int64_t p95_us;       /* nearest-rank P95 of query latency (-1 if failed) */
+  int64_t makespan_us;  /* completion time of the last query */
+  int64_t events;       /* completed LLM calls (= n_calls when ok) */
+  uint64_t digest;      /* order-free checksum of every call's (id, instance, start)
+                           and every query's (id, end) */
+  int32_t slo_met;      /* queries with latency <= T_slo */
+  int32_t n_done;       /* completed queries */
+  int32_t status;       /* HX_OK or HX_ERR_CAPACITY / HX_ERR_STEP_LIMIT */
+  int32_t pad;
+} hx_result;
+
+/* Best point (Sec. 4.3's argmin of P95; the constrained objective keeps
+ * points whose SLO attainment is >= 95%, else the most SLO hits).
+ * Ties go to the lowest point index; failed simulations never win. */
+typedef struct hx_best {
+  int32_t global_point;       /* argmin over points of the sum over traces */
+  int32_t pad;
+  int64_t global_sum_p95;     /* its summed P95 */
+  int64_t global_slo_met;     /* its summed SLO count */
+  int32_t* per_trace_point;   /* caller-owned [n_traces], may be NULL */
+} hx_best;
+
+typedef struct hx_sim hx_sim;
+
+/* Validate and copy traces, cluster and grid to library-owned device memory
+ * and size the per-warp scratch.  On failure *out is NULL. */
+int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cluster,
+                  const hx_grid* grid, const hx_options* opt, hx_sim** out);
+
+/* Replace the trace contents of an existing handle with traces of the same
+ * shapes (n_queries and n_calls per trace), copying host -> device on
+ * `stream`; no allocation. */
+int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream);
+
+/* Enqueue the whole path on `stream` (a cudaStream_t, NULL = legacy default):
+ * per-call preparation, every simulation, the best-point reduction.
+ * Asynchronous; may be called repeatedly. */
+int hx_sim_run(hx_sim* h, void* stream);
+
+/* Wait for the last run and copy n <= n_sims results to host memory. */
+int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n);
+
+/* Wait for the last run and return the best point for `objective`. */
+int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out);
+
+/* Per-call log of recorded simulation `rec_index` (position in
+ * opt.record_sims): instance, dispatch time, SLO budget and start time of
+ * every call of its trace.  Arrays are [n_calls] of that trace. */
+int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us,
+                   int64_t* budget_us, int64_t* start_us, size_t n_calls);
+
+/* Per-call preparation output of trace `trace_index` after a run: Eq. (comp)
+ * per type (est with the believed output, svc with the true output),
+ * [n_calls * 4] type-minor (unused types 0); the mean over instances tbar
+ * [n_calls]; and the query deadline (arrival + T_slo) of each call
+ * [n_calls].  Any pointer may be NULL. */
+int hx_sim_prep(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int32_t* tbar,
+                int64_t* deadline_us, size_t n_calls);
+
+/* Milliseconds of the last run's kernels (prep, simulate, best); needs
+ * opt.timing = 1.  Waits for the run. */
+int hx_sim_timings(hx_sim* h, float* prep_ms, float* sim_ms, float* best_ms);
+
+typedef struct hx_info {
+  int64_t n_sims;
+  int64_t n_calls_total;
+  int64_t n_queries_total;
+  int64_t scratch_bytes;        /* per-warp scratch, all resident warps */
+  int64_t device_bytes;         /* everything the handle holds on the device */
+  int32_t resident_warps;
+  int32_t warps_per_block;
+  int32_t blocks;
+  int32_t smem_per_block;
+} hx_info;
+
+int hx_sim_info(hx_sim* h, hx_info* out);
+
+/* Free everything; NULL is allowed. */
+int hx_sim_destroy(hx_sim* h);
+
+/* The calling thread's last error message ("" if none). */
+const char* hx_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

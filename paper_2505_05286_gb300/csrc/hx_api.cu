@@ -1,0 +1,625 @@
+// hx_api.cu -- the C ABI (include/hxsim.h): input validation, flattening of
+// the traces into device arrays, per-warp scratch sizing and the launches of
+// the preparation, simulation and best-point kernels on the caller's stream.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "hx_device.cuh"
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const std::string& msg) {
+  g_err = msg;
+  return code;
+}
+
+#define HX_CUDA(x)                                                                   \
+  do {                                                                               \
+    cudaError_t e_ = (x);                                                            \
+    if (e_ != cudaSuccess)                                                           \
+      return fail(e_ == cudaErrorMemoryAllocation ? HX_ERR_OOM : HX_ERR_CUDA,        \
+                  std::string(#x) + ": " + cudaGetErrorString(e_));                  \
+  } while (0)
+
+constexpr int64_t kTokMax = int64_t(1) << 20;     // prompt / output tokens per call
+constexpr int64_t kCostMax = int64_t(1) << 28;    // any per-call cost bound, us
+constexpr int64_t kHorizonMax = int64_t(1) << 39; // last arrival + all service, us
+
+int64_t align_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace
+
+struct hx_sim {
+  int32_t n_traces = 0, n_points = 0;
+  int64_t n_sims = 0, n_q = 0, n_c = 0;
+  int32_t max_nq = 0, max_nc = 0, max_kcap = 1;
+  hx::ClusterK ck{};
+  std::vector<int32_t> h_nq, h_nc;
+  // device: inputs
+  int64_t* d_arrival = nullptr;
+  int64_t* d_qcall = nullptr;
+  int64_t* d_q_off = nullptr;
+  int64_t* d_c_off = nullptr;
+  uint8_t* d_k = nullptr;
+  int32_t* d_prompt = nullptr;
+  int32_t* d_out = nullptr;
+  int32_t* d_out_est = nullptr;
+  uint8_t* d_stage = nullptr;
+  uint8_t* d_cand = nullptr;
+  uint8_t* d_retry = nullptr;
+  int64_t* d_alpha = nullptr;
+  int64_t* d_gamma = nullptr;
+  int64_t* d_beta = nullptr;
+  int32_t* d_rho = nullptr;
+  uint8_t* d_lp = nullptr;
+  uint8_t* d_dp = nullptr;
+  // device: derived and outputs
+  hx::CallRec* d_rec = nullptr;
+  hx_result* d_results = nullptr;
+  unsigned long long* d_counter = nullptr;
+  hx::BestCand* d_best_trace = nullptr;
+  hx::BestCand* d_best_global = nullptr;
+  // device: scratch
+  hx::HeapEnt* d_arena = nullptr;
+  uint8_t* d_chains = nullptr;
+  int64_t* d_topk = nullptr;
+  int64_t arena_per_warp = 0, chains_per_warp = 0, topk_per_warp = 0;
+  // device: records
+  int32_t n_record = 0;
+  int64_t rec_stride = 0;
+  int32_t* d_rec_map = nullptr;
+  int32_t* d_rec_inst = nullptr;
+  int64_t* d_rec_enq = nullptr;
+  int64_t* d_rec_budget = nullptr;
+  int64_t* d_rec_start = nullptr;
+  std::vector<int32_t> record_sims;
+  // launch shape
+  int blocks = 0, resident_warps = 0, smem_per_block = 0;
+  int64_t scratch_bytes = 0, device_bytes = 0;
+  cudaStream_t last_stream = nullptr;
+  bool ran = false;
+  bool timing = false;
+  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  std::vector<void*> allocs;
+
+  template <class T>
+  int alloc(T** p, int64_t count) {
+    size_t bytes = (size_t)std::max<int64_t>(count, 1) * sizeof(T);
+    void* q = nullptr;
+    cudaError_t e = cudaMalloc(&q, bytes);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return fail(HX_ERR_OOM, "cudaMalloc of " + std::to_string(bytes) + " bytes: " + cudaGetErrorString(e));
+    }
+    allocs.push_back(q);
+    device_bytes += (int64_t)bytes;
+    *p = static_cast<T*>(q);
+    return HX_OK;
+  }
+
+  ~hx_sim() {
+    for (void* p : allocs) cudaFree(p);
+    for (auto& e : ev)
+      if (e) cudaEventDestroy(e);
+  }
+};
+
+namespace {
+
+int validate_cluster(const hx_cluster* c, int64_t* min_prefill, int64_t* max_decode) {
+  if (!c) return fail(HX_ERR_INVALID, "cluster is NULL");
+  if (c->n_types < 1 || c->n_types > HX_MAX_TYPES) return fail(HX_ERR_INVALID, "n_types must be 1..4");
+  if (c->n_inst < 1 || c->n_inst > HX_MAX_INST) return fail(HX_ERR_INVALID, "n_inst must be 1..64");
+  if (!c->prefill_tok_s || !c->decode_us_tok || !c->slots || !c->inst_type || !c->stage_ref_prompt ||
+      !c->stage_ref_out)
+    return fail(HX_ERR_INVALID, "cluster array is NULL");
+  int64_t mp = INT64_MAX, md = 0;
+  for (int t = 0; t < c->n_types; ++t) {
+    if (c->prefill_tok_s[t] < 1) return fail(HX_ERR_INVALID, "prefill_tok_s must be >= 1");
+    if (c->decode_us_tok[t] < 0) return fail(HX_ERR_INVALID, "decode_us_tok must be >= 0");
+    if (c->slots[t] < 1 || c->slots[t] > HX_MAX_SLOTS) return fail(HX_ERR_INVALID, "slots must be 1..16");
+    mp = std::min<int64_t>(mp, c->prefill_tok_s[t]);
+    md = std::max<int64_t>(md, c->decode_us_tok[t]);
+  }
+  for (int m = 0; m < c->n_inst; ++m)
+    if (c->inst_type[m] >= c->n_types) return fail(HX_ERR_INVALID, "inst_type out of range");
+  if (c->ref_type < 0 || c->ref_type >= c->n_types) return fail(HX_ERR_INVALID, "ref_type out of range");
+  if (c->slo_mult_fp < 0 || c->slo_mult_fp > 16 * HX_SCALE) return fail(HX_ERR_INVALID, "slo_mult_fp must be 0..16*SCALE");
+  if (c->rmax < 0 || c->rmax > HX_MAX_RETRY) return fail(HX_ERR_INVALID, "rmax must be 0..15");
+  for (int s = 0; s < 4; ++s) {
+    const int64_t p = c->stage_ref_prompt[s], o = c->stage_ref_out[s];
+    if (p < 0 || p > kTokMax || o < 0 || o > kTokMax) return fail(HX_ERR_INVALID, "stage reference tokens out of range");
+    if ((p * 1000000 + mp - 1) / mp + o * md >= kCostMax) return fail(HX_ERR_INVALID, "stage reference cost too large");
+  }
+  *min_prefill = mp;
+  *max_decode = md;
+  return HX_OK;
+}
+
+int validate_grid(const hx_grid* g) {
+  if (!g) return fail(HX_ERR_INVALID, "grid is NULL");
+  if (g->n_points < 1) return fail(HX_ERR_INVALID, "n_points must be >= 1");
+  if (!g->alpha_fp || !g->gamma_fp || !g->rho || !g->beta_us2 || !g->local_policy || !g->dispatch_policy)
+    return fail(HX_ERR_INVALID, "grid array is NULL");
+  for (int p = 0; p < g->n_points; ++p) {
+    if (g->alpha_fp[p] < 0 || g->alpha_fp[p] > HX_SCALE) return fail(HX_ERR_INVALID, "alpha_fp must be 0..SCALE");
+    if (g->gamma_fp[p] < 0 || g->gamma_fp[p] > 4 * HX_SCALE) return fail(HX_ERR_INVALID, "gamma_fp must be 0..4*SCALE");
+    if (g->rho[p] < 0 || g->rho[p] > HX_MAX_RETRY) return fail(HX_ERR_INVALID, "rho must be 0..15");
+    if (g->beta_us2[p] < 0 || g->beta_us2[p] > (int64_t(1) << 62)) return fail(HX_ERR_INVALID, "beta_us2 out of range");
+    if (g->local_policy[p] > 1 || g->dispatch_policy[p] > 1) return fail(HX_ERR_INVALID, "unknown policy");
+  }
+  return HX_OK;
+}
+
+int validate_trace(const hx_trace* tr, int ti, const hx_cluster* c, int64_t min_prefill, int64_t max_decode) {
+  const std::string where = "trace " + std::to_string(ti) + ": ";
+  if (tr->n_queries < 0 || tr->n_calls < 0 || tr->n_calls >= (1 << 24))
+    return fail(HX_ERR_INVALID, where + "n_queries/n_calls out of range");
+  if (tr->n_queries > 0 && (!tr->arrival_us || !tr->k || !tr->prompt || !tr->out || !tr->out_est || !tr->stage ||
+                            !tr->cand || !tr->retry))
+    return fail(HX_ERR_INVALID, where + "array is NULL");
+  if (!tr->call_base) return fail(HX_ERR_INVALID, where + "call_base is NULL");
+  if (tr->call_base[0] != 0 || tr->call_base[tr->n_queries] != tr->n_calls)
+    return fail(HX_ERR_INVALID, where + "call_base must run from 0 to n_calls");
+  int64_t horizon = 0;
+  for (int32_t i = 0; i < tr->n_queries; ++i) {
+    if (tr->arrival_us[i] < 0 || (i > 0 && tr->arrival_us[i] < tr->arrival_us[i - 1]))
+      return fail(HX_ERR_INVALID, where + "arrivals must be non-negative and sorted");
+    const int32_t b = tr->call_base[i], e = tr->call_base[i + 1];
+    const int k = tr->k[i];
+    if (k < 1 || k > HX_MAX_K) return fail(HX_ERR_INVALID, where + "k must be 1..8");
+    if (e - b < 2 + k || b < 0 || e > tr->n_calls) return fail(HX_ERR_INVALID, where + "bad call_base");
+    if (tr->stage[b] != HX_STAGE_S || tr->stage[e - 1] != HX_STAGE_E)
+      return fail(HX_ERR_INVALID, where + "a query must start with S and end with E");
+    for (int cd = 0; cd < k; ++cd)
+      if (tr->stage[b + 1 + cd] != HX_STAGE_G || tr->cand[b + 1 + cd] != cd)
+        return fail(HX_ERR_INVALID, where + "S must be followed by G_0..G_{k-1}");
+    int prev_c = -1, prev_r = 0;
+    for (int32_t j = b + 1 + k; j < e - 1; ++j) {
+      const int cd = tr->cand[j], r = tr->retry[j];
+      if (tr->stage[j] != HX_STAGE_C || cd >= k || r < 1 || r > c->rmax)
+        return fail(HX_ERR_INVALID, where + "corrections must be C calls of a candidate with 1 <= retry <= rmax");
+      if (cd == prev_c ? r != prev_r + 1 : (cd < prev_c || r != 1))
+        return fail(HX_ERR_INVALID, where + "corrections must be ordered by (candidate, retry)");
+      prev_c = cd;
+      prev_r = r;
+    }
+    for (int32_t j = b; j < e; ++j) {
+      const int64_t p = tr->prompt[j], o = tr->out[j], oe = tr->out_est[j];
+      if (p < 1 || p > kTokMax || o < 0 || o > kTokMax || oe < 0 || oe > kTokMax)
+        return fail(HX_ERR_INVALID, where + "token counts out of range");
+      const int64_t bound = (p * 1000000 + min_prefill - 1) / min_prefill + std::max(o, oe) * max_decode;
+      if (bound >= kCostMax) return fail(HX_ERR_INVALID, where + "a call's cost exceeds 2^28 us");
+      horizon += bound;
+    }
+  }
+  if (tr->n_queries > 0) horizon += tr->arrival_us[tr->n_queries - 1];
+  if (horizon > kHorizonMax) return fail(HX_ERR_INVALID, where + "time horizon exceeds 2^39 us");
+  return HX_OK;
+}
+
+template <class T>
+int upload(T* dst, const T* src, int64_t count, cudaStream_t s) {
+  if (count <= 0) return HX_OK;
+  HX_CUDA(cudaMemcpyAsync(dst, src, (size_t)count * sizeof(T), cudaMemcpyHostToDevice, s));
+  return HX_OK;
+}
+
+// Copies the per-call and per-query trace arrays of all traces to the device.
+int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
+  std::vector<int64_t> arrival((size_t)h->n_q), qcall((size_t)h->n_q + 1);
+  std::vector<uint8_t> kq((size_t)h->n_q);
+  int64_t qo = 0, co = 0;
+  for (int t = 0; t < h->n_traces; ++t) {
+    const hx_trace& tr = traces[t];
+    for (int32_t i = 0; i < tr.n_queries; ++i) {
+      arrival[qo + i] = tr.arrival_us[i];
+      kq[qo + i] = tr.k[i];
+      qcall[qo + i] = co + tr.call_base[i];
+    }
+    qo += tr.n_queries;
+    co += tr.n_calls;
+  }
+  qcall[h->n_q] = co;
+  int rc;
+  if ((rc = upload(h->d_arrival, arrival.data(), h->n_q, s)) || (rc = upload(h->d_k, kq.data(), h->n_q, s)) ||
+      (rc = upload(h->d_qcall, qcall.data(), h->n_q + 1, s)))
+    return rc;
+  co = 0;
+  for (int t = 0; t < h->n_traces; ++t) {
+    const hx_trace& tr = traces[t];
+    if ((rc = upload(h->d_prompt + co, tr.prompt, tr.n_calls, s)) || (rc = upload(h->d_out + co, tr.out, tr.n_calls, s)) ||
+        (rc = upload(h->d_out_est + co, tr.out_est, tr.n_calls, s)) ||
+        (rc = upload(h->d_stage + co, tr.stage, tr.n_calls, s)) || (rc = upload(h->d_cand + co, tr.cand, tr.n_calls, s)) ||
+        (rc = upload(h->d_retry + co, tr.retry, tr.n_calls, s)))
+      return rc;
+    co += tr.n_calls;
+  }
+  // the host staging vectors die here: the copies must finish first
+  HX_CUDA(cudaStreamSynchronize(s));
+  return HX_OK;
+}
+
+int per_warp_smem(int total_slots) {
+  return (int)align_up((192 + (int64_t)total_slots) * 8 + ((int64_t)total_slots + 320) * 4, 16);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* hx_last_error(void) { return g_err.c_str(); }
+
+int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cluster, const hx_grid* grid,
+                  const hx_options* opt, hx_sim** out) {
+  if (!out) return fail(HX_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  g_err.clear();
+  if (!traces || n_traces < 1) return fail(HX_ERR_INVALID, "need at least one trace");
+  int64_t min_prefill = 0, max_decode = 0;
+  int rc;
+  if ((rc = validate_cluster(cluster, &min_prefill, &max_decode))) return rc;
+  if ((rc = validate_grid(grid))) return rc;
+  for (int t = 0; t < n_traces; ++t)
+    if ((rc = validate_trace(&traces[t], t, cluster, min_prefill, max_decode))) return rc;
+  if (opt && opt->n_record > 0 && !opt->record_sims) return fail(HX_ERR_INVALID, "record_sims is NULL");
+
+  hx_sim* h = new (std::nothrow) hx_sim();
+  if (!h) return fail(HX_ERR_OOM, "host allocation failed");
+  auto bail = [&](int code) {
+    delete h;
+    return code;
+  };
+  h->n_traces = n_traces;
+  h->n_points = grid->n_points;
+  h->n_sims = (int64_t)n_traces * grid->n_points;
+  std::vector<int64_t> q_off(n_traces + 1, 0), c_off(n_traces + 1, 0);
+  for (int t = 0; t < n_traces; ++t) {
+    const int32_t nq = traces[t].n_queries, nc = traces[t].n_calls;
+    h->h_nq.push_back(nq);
+    h->h_nc.push_back(nc);
+    q_off[t + 1] = q_off[t] + nq;
+    c_off[t + 1] = c_off[t] + nc;
+    h->max_nq = std::max(h->max_nq, nq);
+    h->max_nc = std::max(h->max_nc, nc);
+    h->max_kcap = std::max(h->max_kcap, nq - (95 * nq + 99) / 100 + 1);
+  }
+  h->n_q = q_off[n_traces];
+  h->n_c = c_off[n_traces];
+  if (h->n_c >= (int64_t(1) << 31)) return bail(fail(HX_ERR_INVALID, "more than 2^31 calls in total"));
+
+  // cluster constants (kernel parameter)
+  hx::ClusterK& ck = h->ck;
+  ck.n_inst = cluster->n_inst;
+  ck.n_types = cluster->n_types;
+  ck.ref_type = cluster->ref_type;
+  ck.rmax = cluster->rmax;
+  ck.slo_mult_fp = cluster->slo_mult_fp;
+  for (int t = 0; t < HX_MAX_TYPES; ++t) {
+    const bool on = t < cluster->n_types;
+    ck.prefill[t] = on ? cluster->prefill_tok_s[t] : 1;
+    ck.decode[t] = on ? cluster->decode_us_tok[t] : 0;
+    ck.slots[t] = on ? cluster->slots[t] : 0;
+    ck.cnt[t] = 0;
+  }
+  for (int s = 0; s < 4; ++s) {
+    ck.ref_prompt[s] = cluster->stage_ref_prompt[s];
+    ck.ref_out[s] = cluster->stage_ref_out[s];
+  }
+  int base = 0;
+  for (int m = 0; m < HX_MAX_INST; ++m) {
+    const bool on = m < cluster->n_inst;
+    const int ty = on ? cluster->inst_type[m] : 0;
+    ck.inst_type[m] = (uint8_t)ty;
+    ck.inst_slots[m] = on ? (uint8_t)cluster->slots[ty] : 0;
+    ck.slot_base[m] = (uint16_t)base;
+    if (on) {
+      base += cluster->slots[ty];
+      ck.cnt[ty]++;
+    }
+  }
+  ck.total_slots = base;
+  ck.smem_per_warp = per_warp_smem(base);
+
+  int dev = 0;
+  cudaDeviceProp prop;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaGetDeviceProperties(&prop, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return bail(fail(HX_ERR_CUDA, "no CUDA device"));
+  }
+  // device inputs
+  if ((rc = h->alloc(&h->d_arrival, h->n_q)) || (rc = h->alloc(&h->d_k, h->n_q)) ||
+      (rc = h->alloc(&h->d_qcall, h->n_q + 1)) || (rc = h->alloc(&h->d_q_off, n_traces + 1)) ||
+      (rc = h->alloc(&h->d_c_off, n_traces + 1)) || (rc = h->alloc(&h->d_prompt, h->n_c)) ||
+      (rc = h->alloc(&h->d_out, h->n_c)) || (rc = h->alloc(&h->d_out_est, h->n_c)) ||
+      (rc = h->alloc(&h->d_stage, h->n_c)) || (rc = h->alloc(&h->d_cand, h->n_c)) ||
+      (rc = h->alloc(&h->d_retry, h->n_c)) || (rc = h->alloc(&h->d_alpha, h->n_points)) ||
+      (rc = h->alloc(&h->d_gamma, h->n_points)) || (rc = h->alloc(&h->d_beta, h->n_points)) ||
+      (rc = h->alloc(&h->d_rho, h->n_points)) || (rc = h->alloc(&h->d_lp, h->n_points)) ||
+      (rc = h->alloc(&h->d_dp, h->n_points)) || (rc = h->alloc(&h->d_rec, h->n_c)) ||
+      (rc = h->alloc(&h->d_results, h->n_sims)) || (rc = h->alloc(&h->d_counter, 1)) ||
+      (rc = h->alloc(&h->d_best_trace, 2 * (int64_t)n_traces)) || (rc = h->alloc(&h->d_best_global, 2)))
+    return bail(rc);
+  cudaStream_t s0 = nullptr;
+  if ((rc = upload_traces(h, traces, s0)) || (rc = upload(h->d_q_off, q_off.data(), n_traces + 1, s0)) ||
+      (rc = upload(h->d_c_off, c_off.data(), n_traces + 1, s0)) ||
+      (rc = upload(h->d_alpha, grid->alpha_fp, h->n_points, s0)) ||
+      (rc = upload(h->d_gamma, grid->gamma_fp, h->n_points, s0)) ||
+      (rc = upload(h->d_beta, grid->beta_us2, h->n_points, s0)) || (rc = upload(h->d_rho, grid->rho, h->n_points, s0)) ||
+      (rc = upload(h->d_lp, grid->local_policy, h->n_points, s0)) ||
+      (rc = upload(h->d_dp, grid->dispatch_policy, h->n_points, s0)))
+    return bail(rc);
+
+  // launch shape of the simulation kernel and its per-warp scratch
+  h->smem_per_block = hx::kWarpsPerBlock * ck.smem_per_warp;
+  if (cudaFuncSetAttribute(hx::hx_sim_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, h->smem_per_block) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return bail(fail(HX_ERR_CUDA, "cannot reserve shared memory for the simulation kernel"));
+  }
+  int bps = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, hx::hx_sim_kernel, hx::kWarpsPerBlock * 32,
+                                                    h->smem_per_block) != cudaSuccess || bps < 1) {
+    cudaGetLastError();
+    return bail(fail(HX_ERR_CUDA, "simulation kernel does not fit on an SM"));
+  }
+  int64_t blocks = (int64_t)bps * prop.multiProcessorCount;
+  if (opt && opt->max_resident_warps > 0)
+    blocks = std::min<int64_t>(blocks, std::max<int64_t>(1, opt->max_resident_warps / hx::kWarpsPerBlock));
+  blocks = std::min<int64_t>(blocks, (h->n_sims + hx::kWarpsPerBlock - 1) / hx::kWarpsPerBlock);
+  h->blocks = (int)std::max<int64_t>(blocks, 1);
+  h->resident_warps = h->blocks * hx::kWarpsPerBlock;
+  // heap arena: doubling regions of 16, 32, ... entries per instance total at
+  // most 4 * (requests ever queued) + 16 * instances
+  h->arena_per_warp = 4 * (int64_t)h->max_nc + 16 * HX_MAX_INST;
+  h->chains_per_warp = align_up(std::max(h->max_nq, 1), 256);
+  h->topk_per_warp = align_up(h->max_kcap, 32);
+  const int64_t w = h->resident_warps;
+  if ((rc = h->alloc(&h->d_arena, w * h->arena_per_warp)) || (rc = h->alloc(&h->d_chains, w * h->chains_per_warp)) ||
+      (rc = h->alloc(&h->d_topk, w * h->topk_per_warp)))
+    return bail(rc);
+  h->scratch_bytes = w * (h->arena_per_warp * (int64_t)sizeof(hx::HeapEnt) + h->chains_per_warp +
+                          h->topk_per_warp * (int64_t)sizeof(int64_t));
+
+  // per-call logs of selected simulations
+  if (opt && opt->n_record > 0) {
+    h->n_record = opt->n_record;
+    h->rec_stride = std::max(h->max_nc, 1);
+    std::vector<int32_t> map((size_t)h->n_sims, -1);
+    for (int j = 0; j < opt->n_record; ++j) {
+      const int32_t sim = opt->record_sims[j];
+      if (sim < 0 || sim >= h->n_sims || map[sim] >= 0)
+        return bail(fail(HX_ERR_INVALID, "record_sims must be distinct valid sim indices"));
+      map[sim] = j;
+      h->record_sims.push_back(sim);
+    }
+    const int64_t n = (int64_t)h->n_record * h->rec_stride;
+    if ((rc = h->alloc(&h->d_rec_map, h->n_sims)) || (rc = h->alloc(&h->d_rec_inst, n)) ||
+        (rc = h->alloc(&h->d_rec_enq, n)) || (rc = h->alloc(&h->d_rec_budget, n)) ||
+        (rc = h->alloc(&h->d_rec_start, n)) || (rc = upload(h->d_rec_map, map.data(), h->n_sims, s0)))
+      return bail(rc);
+    if (cudaStreamSynchronize(s0) != cudaSuccess) return bail(fail(HX_ERR_CUDA, "record map upload failed"));
+  }
+  if (opt && opt->timing) {
+    h->timing = true;
+    for (auto& e : h->ev)
+      if (cudaEventCreate(&e) != cudaSuccess) return bail(fail(HX_ERR_CUDA, "cudaEventCreate failed"));
+  }
+  if (cudaDeviceSynchronize() != cudaSuccess) return bail(fail(HX_ERR_CUDA, "upload failed"));
+  *out = h;
+  return HX_OK;
+}
+
+int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream) {
+  if (!h || !traces) return fail(HX_ERR_INVALID, "NULL argument");
+  if (n_traces != h->n_traces) return fail(HX_ERR_INVALID, "trace count differs from the handle's");
+  for (int t = 0; t < n_traces; ++t)
+    if (traces[t].n_queries != h->h_nq[t] || traces[t].n_calls != h->h_nc[t])
+      return fail(HX_ERR_INVALID, "trace shapes differ from the handle's");
+  // same validation as create, against the handle's cluster bounds
+  int64_t min_prefill = INT64_MAX, max_decode = 0;
+  for (int t = 0; t < h->ck.n_types; ++t) {
+    min_prefill = std::min<int64_t>(min_prefill, h->ck.prefill[t]);
+    max_decode = std::max<int64_t>(max_decode, h->ck.decode[t]);
+  }
+  hx_cluster c{};
+  c.rmax = h->ck.rmax;
+  for (int t = 0; t < n_traces; ++t) {
+    int rc = validate_trace(&traces[t], t, &c, min_prefill, max_decode);
+    if (rc) return rc;
+  }
+  return upload_traces(h, traces, static_cast<cudaStream_t>(stream));
+}
+
+int hx_sim_run(hx_sim* h, void* stream) {
+  if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  hx::PrepArgs pa;
+  pa.arrival = h->d_arrival;
+  pa.kq = h->d_k;
+  pa.qcall = h->d_qcall;
+  pa.q_off = h->d_q_off;
+  pa.c_off = h->d_c_off;
+  pa.prompt = h->d_prompt;
+  pa.out = h->d_out;
+  pa.out_est = h->d_out_est;
+  pa.stage = h->d_stage;
+  pa.cand = h->d_cand;
+  pa.retry = h->d_retry;
+  pa.n_queries = h->n_q;
+  pa.n_traces = h->n_traces;
+  pa.rec = h->d_rec;
+  pa.work_counter = h->d_counter;
+
+  hx::SimArgs sa;
+  sa.rec = h->d_rec;
+  sa.arrival = h->d_arrival;
+  sa.qcall = h->d_qcall;
+  sa.q_off = h->d_q_off;
+  sa.c_off = h->d_c_off;
+  sa.alpha = h->d_alpha;
+  sa.gamma = h->d_gamma;
+  sa.rho = h->d_rho;
+  sa.beta = h->d_beta;
+  sa.lpol = h->d_lp;
+  sa.dpol = h->d_dp;
+  sa.n_points = h->n_points;
+  sa.n_traces = h->n_traces;
+  sa.n_sims = h->n_sims;
+  sa.results = h->d_results;
+  sa.work_counter = h->d_counter;
+  sa.arena = h->d_arena;
+  sa.arena_per_warp = h->arena_per_warp;
+  sa.chains = h->d_chains;
+  sa.chains_per_warp = h->chains_per_warp;
+  sa.topk = h->d_topk;
+  sa.topk_per_warp = h->topk_per_warp;
+  sa.rec_map = h->d_rec_map;
+  sa.rec_inst = h->d_rec_inst;
+  sa.rec_enq = h->d_rec_enq;
+  sa.rec_budget = h->d_rec_budget;
+  sa.rec_start = h->d_rec_start;
+  sa.rec_stride = h->rec_stride;
+
+  hx::BestArgs ba;
+  ba.results = h->d_results;
+  ba.q_off = h->d_q_off;
+  ba.n_traces = h->n_traces;
+  ba.n_points = h->n_points;
+  ba.per_trace = h->d_best_trace;
+  ba.global = h->d_best_global;
+
+  const int prep_blocks = (int)std::max<int64_t>(1, (h->n_q + 255) / 256);
+  if (h->timing) HX_CUDA(cudaEventRecord(h->ev[0], s));
+  hx::hx_prep_kernel<<<prep_blocks, 256, 0, s>>>(pa, h->ck);
+  HX_CUDA(cudaGetLastError());
+  if (h->timing) HX_CUDA(cudaEventRecord(h->ev[1], s));
+  hx::hx_sim_kernel<<<h->blocks, hx::kWarpsPerBlock * 32, h->smem_per_block, s>>>(sa, h->ck);
+  HX_CUDA(cudaGetLastError());
+  if (h->timing) HX_CUDA(cudaEventRecord(h->ev[2], s));
+  hx::hx_best_kernel<<<h->n_traces + 1, 256, 0, s>>>(ba);
+  HX_CUDA(cudaGetLastError());
+  if (h->timing) HX_CUDA(cudaEventRecord(h->ev[3], s));
+  h->last_stream = s;
+  h->ran = true;
+  return HX_OK;
+}
+
+int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n) {
+  if (!h || !host_out) return fail(HX_ERR_INVALID, "NULL argument");
+  if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
+  if ((int64_t)n > h->n_sims) return fail(HX_ERR_INVALID, "n exceeds the number of simulations");
+  HX_CUDA(cudaStreamSynchronize(h->last_stream));
+  HX_CUDA(cudaMemcpy(host_out, h->d_results, n * sizeof(hx_result), cudaMemcpyDeviceToHost));
+  return HX_OK;
+}
+
+int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out) {
+  if (!h || !out) return fail(HX_ERR_INVALID, "NULL argument");
+  if (objective != HX_OBJ_P95 && objective != HX_OBJ_P95_SLO95) return fail(HX_ERR_INVALID, "unknown objective");
+  if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
+  HX_CUDA(cudaStreamSynchronize(h->last_stream));
+  hx::BestCand g[2];
+  HX_CUDA(cudaMemcpy(g, h->d_best_global, sizeof(g), cudaMemcpyDeviceToHost));
+  const bool gv = g[objective].flags & 1;
+  out->global_point = gv ? g[objective].p : -1;
+  out->pad = 0;
+  out->global_sum_p95 = gv ? g[objective].p95 : -1;
+  out->global_slo_met = gv ? g[objective].slo : -1;
+  if (out->per_trace_point) {
+    std::vector<hx::BestCand> pt((size_t)2 * h->n_traces);
+    HX_CUDA(cudaMemcpy(pt.data(), h->d_best_trace, pt.size() * sizeof(hx::BestCand), cudaMemcpyDeviceToHost));
+    for (int t = 0; t < h->n_traces; ++t) {
+      const hx::BestCand& b = pt[(size_t)2 * t + objective];
+      out->per_trace_point[t] = (b.flags & 1) ? b.p : -1;
+    }
+  }
+  return HX_OK;
+}
+
+int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us, int64_t* budget_us,
+                   int64_t* start_us, size_t n_calls) {
+  if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
+  if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
+  if (rec_index < 0 || rec_index >= h->n_record) return fail(HX_ERR_INVALID, "rec_index out of range");
+  const int t = (int)(h->record_sims[rec_index] / h->n_points);
+  if ((int64_t)n_calls != h->h_nc[t]) return fail(HX_ERR_INVALID, "n_calls differs from the trace's");
+  HX_CUDA(cudaStreamSynchronize(h->last_stream));
+  const int64_t o = (int64_t)rec_index * h->rec_stride;
+  if (n_calls == 0) return HX_OK;
+  if (inst) HX_CUDA(cudaMemcpy(inst, h->d_rec_inst + o, n_calls * sizeof(int32_t), cudaMemcpyDeviceToHost));
+  if (enq_us) HX_CUDA(cudaMemcpy(enq_us, h->d_rec_enq + o, n_calls * sizeof(int64_t), cudaMemcpyDeviceToHost));
+  if (budget_us) HX_CUDA(cudaMemcpy(budget_us, h->d_rec_budget + o, n_calls * sizeof(int64_t), cudaMemcpyDeviceToHost));
+  if (start_us) HX_CUDA(cudaMemcpy(start_us, h->d_rec_start + o, n_calls * sizeof(int64_t), cudaMemcpyDeviceToHost));
+  return HX_OK;
+}
+
+int hx_sim_prep(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int32_t* tbar, int64_t* deadline_us,
+                size_t n_calls) {
+  if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
+  if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
+  if (trace_index < 0 || trace_index >= h->n_traces) return fail(HX_ERR_INVALID, "trace_index out of range");
+  if ((int64_t)n_calls != h->h_nc[trace_index]) return fail(HX_ERR_INVALID, "n_calls differs from the trace's");
+  HX_CUDA(cudaStreamSynchronize(h->last_stream));
+  if (n_calls == 0) return HX_OK;
+  int64_t off = 0;
+  for (int t = 0; t < trace_index; ++t) off += h->h_nc[t];
+  std::vector<hx::CallRec> recs(n_calls);
+  HX_CUDA(cudaMemcpy(recs.data(), h->d_rec + off, n_calls * sizeof(hx::CallRec), cudaMemcpyDeviceToHost));
+  for (size_t j = 0; j < n_calls; ++j) {
+    for (int ty = 0; ty < 4; ++ty) {
+      if (est) est[4 * j + ty] = recs[j].est[ty];
+      if (svc) svc[4 * j + ty] = recs[j].svc[ty];
+    }
+    if (tbar) tbar[j] = recs[j].tbar;
+    if (deadline_us) deadline_us[j] = recs[j].deadline;
+  }
+  return HX_OK;
+}
+
+int hx_sim_timings(hx_sim* h, float* prep_ms, float* sim_ms, float* best_ms) {
+  if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
+  if (!h->timing) return fail(HX_ERR_STATE, "created without opt.timing");
+  if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
+  HX_CUDA(cudaEventSynchronize(h->ev[3]));
+  float a = 0, b = 0, c = 0;
+  HX_CUDA(cudaEventElapsedTime(&a, h->ev[0], h->ev[1]));
+  HX_CUDA(cudaEventElapsedTime(&b, h->ev[1], h->ev[2]));
+  HX_CUDA(cudaEventElapsedTime(&c, h->ev[2], h->ev[3]));
+  if (prep_ms) *prep_ms = a;
+  if (sim_ms) *sim_ms = b;
+  if (best_ms) *best_ms = c;
+  return HX_OK;
+}
+
+int hx_sim_info(hx_sim* h, hx_info* out) {
+  if (!h || !out) return fail(HX_ERR_INVALID, "NULL argument");
+  out->n_sims = h->n_sims;
+  out->n_calls_total = h->n_c;
+  out->n_queries_total = h->n_q;
+  out->scratch_bytes = h->scratch_bytes;
+  out->device_bytes = h->device_bytes;
+  out->resident_warps = h->resident_warps;
+  out->warps_per_block = hx::kWarpsPerBlock;
+  out->blocks = h->blocks;
+  out->smem_per_block = h->smem_per_block;
+  return HX_OK;
+}
+
+int hx_sim_destroy(hx_sim* h) {
+  if (!h) return HX_OK;
+  if (h->ran && h->last_stream) cudaStreamSynchronize(h->last_stream);
+  cudaDeviceSynchronize();
+  delete h;
+  return HX_OK;
+}
+
+}  // extern "C"

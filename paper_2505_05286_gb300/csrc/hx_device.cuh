@@ -1,0 +1,132 @@
+// hx_device.cuh -- device-side data layout and kernels of the batched
+// HexGen-Flow scheduler simulation (arXiv 2505.05286, Sec. 4) for sm_103a.
+//
+//   hx_prep_kernel  : per query, Eq. (comp) per call and instance type, the
+//                     mean cost tbar of Sec. 4.2, workflow successor links
+//                     (Sec. 2.1) and the query deadline (SLO of Sec. 5.1);
+//                     writes one 64-byte record per call.
+//   hx_sim_kernel   : persistent; one warp runs one (trace, point) discrete
+//                     event simulation of the workload-balanced dispatcher
+//                     (Sec. 4.1) and the urgency queues (Sec. 4.2), and
+//                     reduces it to P95 / SLO count / digest (Sec. 4.3).
+//   hx_best_kernel  : argmin of the P95 objective per trace and over the grid.
+#pragma once
+
+#include <stdint.h>
+
+#include "hxsim.h"
+
+namespace hx {
+
+constexpr int64_t kScale = 1000000;       // fixed point of alpha, gamma, slo_mult
+constexpr int64_t kUsPerS = 1000000;      // prefill throughput is per second
+constexpr int64_t kRewardCap = (int64_t(1) << 43) - 1;
+constexpr uint64_t kKeyInf = ~0ull;
+constexpr int64_t kTimeInf = INT64_MAX;
+constexpr int kWarpsPerBlock = 4;
+constexpr unsigned kFull = 0xffffffffu;
+constexpr uint64_t kArrivalTag = 64;      // event-key tag: after every instance
+
+// One call as the simulator reads it: 64 bytes, 16-byte aligned.
+struct __align__(16) CallRec {
+  int32_t est[4];     // Eq. (comp) with the believed output length, per type
+  int32_t svc[4];     // the same with the true output length (service time)
+  int64_t deadline;   // query arrival + T_slo
+  int64_t arrival;    // query arrival
+  int32_t tbar;       // mean of est over the instances
+  int32_t next;       // S: unused; G/C: next correction's id, or ~(E's id) at chain end
+  int32_t qid;        // query index within the trace
+  uint8_t stage, u, k, pad;  // stage, corrections done incl. this call, k of the query
+};
+static_assert(sizeof(CallRec) == 64, "CallRec is one 64-byte unit");
+
+// Local-queue entry: priority key (higher first) and request id (lower first).
+struct __align__(16) HeapEnt {
+  long long key;
+  int rid;
+  int pad;
+};
+
+// Cluster description passed by value (kernel parameter space).
+struct ClusterK {
+  int32_t n_inst, n_types, ref_type, rmax;
+  int64_t slo_mult_fp;
+  int32_t prefill[HX_MAX_TYPES], decode[HX_MAX_TYPES], slots[HX_MAX_TYPES], cnt[HX_MAX_TYPES];
+  int32_t ref_prompt[4], ref_out[4];
+  int32_t total_slots;
+  int32_t smem_per_warp;
+  uint8_t inst_type[HX_MAX_INST];
+  uint8_t inst_slots[HX_MAX_INST];
+  uint16_t slot_base[HX_MAX_INST];
+};
+
+struct PrepArgs {
+  const int64_t* arrival;   // [Q]
+  const uint8_t* kq;        // [Q]
+  const int64_t* qcall;     // [Q + 1] first call (global index) of each query
+  const int64_t* q_off;     // [T + 1]
+  const int64_t* c_off;     // [T + 1]
+  const int32_t* prompt;
+  const int32_t* out;
+  const int32_t* out_est;
+  const uint8_t* stage;
+  const uint8_t* cand;
+  const uint8_t* retry;
+  int64_t n_queries;
+  int32_t n_traces;
+  CallRec* rec;             // [C]
+  unsigned long long* work_counter;
+};
+
+struct SimArgs {
+  const CallRec* rec;
+  const int64_t* arrival;
+  const int64_t* qcall;
+  const int64_t* q_off;
+  const int64_t* c_off;
+  const int64_t* alpha;
+  const int64_t* gamma;
+  const int32_t* rho;
+  const int64_t* beta;
+  const uint8_t* lpol;
+  const uint8_t* dpol;
+  int32_t n_points;
+  int32_t n_traces;
+  int64_t n_sims;
+  hx_result* results;
+  unsigned long long* work_counter;
+  HeapEnt* arena;           // per resident warp: arena_per_warp entries
+  int64_t arena_per_warp;
+  uint8_t* chains;          // per resident warp: chains_per_warp bytes
+  int64_t chains_per_warp;
+  int64_t* topk;            // per resident warp: topk_per_warp latencies
+  int64_t topk_per_warp;
+  const int32_t* rec_map;   // [n_sims] record slot or -1; NULL when not recording
+  int32_t* rec_inst;
+  int64_t* rec_enq;
+  int64_t* rec_budget;
+  int64_t* rec_start;
+  int64_t rec_stride;
+};
+
+struct BestCand {
+  int64_t p95;
+  int64_t slo;
+  int32_t p;
+  int32_t flags;  // bit0 valid, bit1 feasible
+};
+
+struct BestArgs {
+  const hx_result* results;
+  const int64_t* q_off;
+  int32_t n_traces;
+  int32_t n_points;
+  BestCand* per_trace;      // [T * 2]
+  BestCand* global;         // [2]
+};
+
+__global__ void hx_prep_kernel(PrepArgs a, ClusterK c);
+__global__ void hx_sim_kernel(SimArgs a, ClusterK c);
+__global__ void hx_best_kernel(BestArgs a);
+
+}  // namespace hx

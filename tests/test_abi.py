@@ -1,0 +1,146 @@
+"""The C ABI without a GPU: the library builds for sm_103a, loads, exports
+every function include/hxsim.h declares, its structs match the binding's
+layout, and malformed inputs are rejected before any device work."""
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+import pytest
+
+from paper_2505_05286_gb300 import build as B
+from paper_2505_05286_gb300 import hxsim as H
+from paper_2505_05286_gb300 import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return H.load()
+
+
+def test_exports_every_declared_function(lib):
+    names = H.declared_functions()
+    assert len(names) >= 11
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in include/hxsim.h but not exported"
+
+
+_PROBE = r"""
+#include <stdio.h>
+#include <stddef.h>
+#include "hxsim.h"
+#define F(T, f) printf(#T "." #f " %zu %zu\n", offsetof(T, f), sizeof(((T*)0)->f));
+#define S(T) printf(#T " %zu\n", sizeof(T));
+int main(void) {
+  S(hx_trace) F(hx_trace, n_queries) F(hx_trace, arrival_us) F(hx_trace, retry)
+  S(hx_cluster) F(hx_cluster, n_inst) F(hx_cluster, inst_type) F(hx_cluster, slo_mult_fp) F(hx_cluster, rmax)
+  F(hx_cluster, stage_ref_out)
+  S(hx_grid) F(hx_grid, alpha_fp) F(hx_grid, dispatch_policy)
+  S(hx_options) F(hx_options, record_sims) F(hx_options, timing)
+  S(hx_result) F(hx_result, digest) F(hx_result, status)
+  S(hx_best) F(hx_best, global_sum_p95) F(hx_best, per_trace_point)
+  S(hx_info) F(hx_info, resident_warps) F(hx_info, smem_per_block)
+  return 0;
+}
+"""
+
+
+def test_struct_layout_matches_binding(tmp_path):
+    src = tmp_path / "probe.c"
+    src.write_text(_PROBE)
+    exe = tmp_path / "probe"
+    subprocess.check_call(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)])
+    got = {}
+    for line in subprocess.check_output([str(exe)], text=True).splitlines():
+        parts = line.split()
+        got[parts[0]] = tuple(int(x) for x in parts[1:])
+    structs = {"hx_trace": H.hx_trace, "hx_cluster": H.hx_cluster, "hx_grid": H.hx_grid,
+               "hx_options": H.hx_options, "hx_best": H.hx_best, "hx_info": H.hx_info}
+    for key, val in got.items():
+        if "." in key:
+            sname, field = key.split(".")
+            if sname == "hx_result":
+                assert H.RESULT_DTYPE.fields[field][1] == val[0]
+                continue
+            ct = structs[sname]
+            assert getattr(ct, field).offset == val[0], key
+            assert getattr(ct, field).size == val[1], key
+        elif key == "hx_result":
+            assert H.RESULT_DTYPE.itemsize == val[0]
+        else:
+            assert ctypes.sizeof(structs[key]) == val[0], key
+
+
+def _create(lib, traces, cluster, grid):
+    t = H._Traces(traces)
+    c = cluster
+    cc = [np.ascontiguousarray(x) for x in (c.prefill_tok_s.astype(np.int32), c.decode_us_tok.astype(np.int32),
+                                            c.slots.astype(np.int32), c.inst_type.astype(np.uint8),
+                                            c.stage_ref_prompt.astype(np.int32), c.stage_ref_out.astype(np.int32))]
+    hc = H.hx_cluster(len(cc[0]), H._p(cc[0]), H._p(cc[1]), H._p(cc[2]), len(cc[3]), H._p(cc[3]), c.ref_type,
+                      c.slo_mult_fp, c.rmax, H._p(cc[4]), H._p(cc[5]))
+    g = grid
+    gc = [np.ascontiguousarray(g.alpha_fp, np.int64), np.ascontiguousarray(g.gamma_fp, np.int64),
+          np.ascontiguousarray(g.rho, np.int32), np.ascontiguousarray(g.beta_us2, np.int64),
+          np.ascontiguousarray(g.local_policy, np.uint8), np.ascontiguousarray(g.dispatch_policy, np.uint8)]
+    hg = H.hx_grid(len(gc[0]), *[H._p(x) for x in gc])
+    h = ctypes.c_void_p()
+    rc = lib.hx_sim_create(t.arr, len(traces), ctypes.byref(hc), ctypes.byref(hg), None, ctypes.byref(h))
+    return rc, lib.hx_last_error().decode(), h
+
+
+def _copy_trace(tr):
+    return W.Trace(*[getattr(tr, f).copy() for f in ("arrival_us", "k", "call_base", "prompt", "out", "out_est",
+                                                      "stage", "cand", "retry")])
+
+
+def test_rejects_malformed_inputs_without_device_work(lib):
+    wl = W.make_workload(0, n_queries=20)
+    tr = wl.traces[0]
+    cases = []
+    t1 = _copy_trace(tr)
+    t1.arrival_us[3] = t1.arrival_us[2] - 1
+    cases.append(("unsorted arrivals", [t1], wl.cluster, wl.grid, "sorted"))
+    t2 = _copy_trace(tr)
+    t2.stage[1] = W.STAGE_E
+    cases.append(("broken workflow", [t2], wl.cluster, wl.grid, "S must be followed"))
+    t3 = _copy_trace(tr)
+    t3.prompt[0] = 0
+    cases.append(("zero prompt", [t3], wl.cluster, wl.grid, "token"))
+    t4 = _copy_trace(tr)
+    t4.k[0] = 9
+    cases.append(("k > 8", [t4], wl.cluster, wl.grid, "k must be"))
+    g = W.Grid(wl.grid.alpha_fp.copy(), wl.grid.gamma_fp.copy(), wl.grid.rho.copy(), wl.grid.beta_us2.copy(),
+               wl.grid.local_policy.copy(), wl.grid.dispatch_policy.copy())
+    g.alpha_fp[0] = W.SCALE + 1
+    cases.append(("alpha > 1", [tr], wl.cluster, g, "alpha"))
+    c = wl.cluster
+    c2 = W.Cluster(c.prefill_tok_s, c.decode_us_tok, np.array([8, 17], np.int32), c.inst_type, c.ref_type,
+                   c.slo_mult_fp, c.rmax, c.stage_ref_prompt, c.stage_ref_out)
+    cases.append(("17 slots", [tr], c2, wl.grid, "slots"))
+    c3 = W.Cluster(c.prefill_tok_s, c.decode_us_tok, c.slots, np.zeros(65, np.uint8), c.ref_type, c.slo_mult_fp,
+                   c.rmax, c.stage_ref_prompt, c.stage_ref_out)
+    cases.append(("65 instances", [tr], c3, wl.grid, "n_inst"))
+    t5 = _copy_trace(tr)
+    t5.arrival_us[:] += 1 << 40
+    cases.append(("horizon", [t5], wl.cluster, wl.grid, "horizon"))
+    for name, trs, cl, gr, msg in cases:
+        rc, err, h = _create(lib, trs, cl, gr)
+        assert rc == H.HX_ERR_INVALID, name
+        assert msg in err, (name, err)
+        assert not h.value
+
+
+def test_null_safety(lib):
+    assert lib.hx_sim_destroy(None) == H.HX_OK
+    assert lib.hx_sim_run(None, None) == H.HX_ERR_INVALID
+    assert lib.hx_sim_results(None, None, 0) == H.HX_ERR_INVALID
+    assert lib.hx_last_error().decode() != ""
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(ImportError):
+        H.load(str(tmp_path / "nope.so"))

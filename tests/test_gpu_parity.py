@@ -1,0 +1,280 @@
+"""CUDA path vs the CPU oracle, bit for bit, through the C ABI.
+
+Everything here is integer work, so the bar is exact equality: per-call
+instance, dispatch time, SLO budget and start time (full logs), and per
+simulation P95, makespan, completed calls, digest, SLO count and status; the
+best points of Sec. 4.3 likewise.  Small cases compare every simulation;
+the full-size workloads compare a seeded sample of simulations plus
+properties that hold at any size.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2505_05286_gb300 import build as B
+from paper_2505_05286_gb300 import hxsim as H
+from paper_2505_05286_gb300 import workloads as W
+from tests import cases
+
+pytestmark = pytest.mark.gpu
+
+NPROC = max(1, min(16, os.cpu_count() or 1))
+FIELDS = ["p95_us", "makespan_us", "events", "digest", "slo_met", "n_done", "status"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    B.build()
+    H.load()
+
+
+def gpu(wl, record=(), **kw):
+    sim = H.Sim(wl.traces, wl.cluster, wl.grid, record_sims=record, **kw)
+    sim.run()
+    return sim
+
+
+def assert_same(g, o, what=""):
+    for f in FIELDS:
+        bad = np.nonzero(g[f] != o[f])[0]
+        assert bad.size == 0, f"{what} field {f} differs at {bad[:8].tolist()}: gpu {g[f][bad[:4]]} oracle {o[f][bad[:4]]}"
+
+
+def assert_logs(sim, wl, j):
+    s = sim.record_sims[j]
+    P = wl.grid.n_points
+    tr = wl.traces[s // P]
+    _, lo = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, s % P), log=True)
+    lg = sim.records(j)
+    for f in ("inst", "enq", "budget", "start"):
+        bad = np.nonzero(lg[f] != lo[f])[0]
+        assert bad.size == 0, f"sim {s}: {f} differs first at call {bad[:5].tolist()}"
+
+
+def oracle_results(wl, sims):
+    return oracle.run(wl, sims, procs=NPROC)
+
+
+def check_best(sim, wl, res):
+    nq = [t.n_queries for t in wl.traces]
+    for obj in (W.OBJ_P95, W.OBJ_P95_SLO95):
+        gp, gs, per = oracle.best(res, len(wl.traces), wl.grid.n_points, nq, obj)
+        bp, bs, _, bper = sim.best(obj)
+        assert (bp, bs) == (gp, gs) and bper.tolist() == per.tolist(), f"objective {obj}"
+
+
+# ------------------------------------------------------------------ hand cases
+@pytest.mark.parametrize("name", sorted(cases.load_golden("hand_cases.json")["cases"].keys()))
+def test_hand_case(name):
+    tr, cl, exp = cases.hand_case(name)
+    grid = cases.grid_from_points([exp["point"]])
+    wl = W.Workload(name, [tr], cl, grid, W.OBJ_P95)
+    sim = gpu(wl, record=[0])
+    r = sim.results()[0]
+    lg = sim.records(0)
+    assert r["status"] == 0
+    assert lg["inst"].tolist() == exp["inst"]
+    assert lg["start"].tolist() == exp["start"]
+    if "budget" in exp:
+        assert lg["budget"].tolist() == exp["budget"]
+    assert int(r["p95_us"]) == exp["p95_us"] and int(r["slo_met"]) == exp["slo_met"]
+    assert int(r["makespan_us"]) == exp["makespan_us"]
+    sim.close()
+
+
+# ---------------------------------------------------------------- preparation
+@pytest.mark.parametrize("cfg,nt,nq", [(0, None, None), (2, 2, 300), (3, 1, 500), (4, 2, 300)])
+def test_prep_matches_oracle(cfg, nt, nq):
+    wl = W.make_workload(cfg, n_traces=nt, n_queries=nq)
+    sim = gpu(wl)
+    T = wl.cluster.n_types
+    for t, tr in enumerate(wl.traces):
+        g = sim.prep(t)
+        o = oracle.prep(tr, wl.cluster)
+        assert (g["est"][:, :T] == o["est"]).all() and (g["svc"][:, :T] == o["svc"]).all()
+        assert (g["tbar"] == o["tbar"]).all()
+        qid = np.repeat(np.arange(tr.n_queries), np.diff(tr.call_base))
+        assert (g["deadline"] == tr.arrival_us[qid] + o["t_slo"][qid]).all()
+    sim.close()
+
+
+# ------------------------------------------------------------- small, complete
+def test_recipe0_every_sim_and_every_call():
+    wl = W.make_workload(0)
+    sim = gpu(wl, record=range(wl.n_sims))
+    g = sim.results()
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(g, o, "recipe 0")
+    for j in range(wl.n_sims):
+        assert_logs(sim, wl, j)
+    check_best(sim, wl, o)
+    golden = cases.load_golden("cfg0_oracle.json")
+    assert [int(x) for x in g["digest"]] == [r["digest"] for r in golden["results"]]
+    sim.close()
+
+
+REDUCED = [
+    (1, 2, 400, 6),
+    (2, 2, 300, 6),
+    (3, 1, 300, 6),
+    (4, 1, 200, 6),
+]
+
+
+@pytest.mark.parametrize("cfg,nt,nq,nrec", REDUCED)
+def test_reduced_recipes_every_sim(cfg, nt, nq, nrec):
+    wl = W.make_workload(cfg, n_traces=nt, n_queries=nq)
+    rng = np.random.default_rng(cfg)
+    rec = sorted(rng.choice(wl.n_sims, size=nrec, replace=False).tolist() + [wl.n_sims - 1])
+    rec = sorted(set(rec))
+    sim = gpu(wl, record=rec)
+    g = sim.results()
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(g, o, f"recipe {cfg}")
+    for j in range(len(rec)):
+        assert_logs(sim, wl, j)
+    check_best(sim, wl, o)
+    sim.close()
+
+
+@pytest.mark.parametrize("local,dispatch", [(W.POLICY_FCFS, W.DISPATCH_WB), (W.POLICY_PQ, W.DISPATCH_RR),
+                                            (W.POLICY_FCFS, W.DISPATCH_RR)])
+def test_policy_variants(local, dispatch):
+    wl = W.make_workload(1, n_traces=2, n_queries=300)
+    g0 = wl.grid
+    wl.grid = W.Grid(g0.alpha_fp, g0.gamma_fp, g0.rho, g0.beta_us2, np.full(g0.n_points, local, np.uint8),
+                     np.full(g0.n_points, dispatch, np.uint8))
+    sim = gpu(wl, record=[0, 77])
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(sim.results(), o, "policies")
+    assert_logs(sim, wl, 0)
+    assert_logs(sim, wl, 1)
+    sim.close()
+
+
+def test_overload_long_queues():
+    """alpha near 1 on recipe 4 routes nearly everything to one instance: its
+    local queue grows to thousands and its heap is re-homed many times."""
+    wl = W.make_workload(4, n_traces=1, n_queries=3000)
+    pts = list(range(1024 - 16, 1024)) + list(range(896 - 8, 896)) + [0, 5, 300]
+    wl.grid = W.subset_grid(wl.grid, pts)
+    sim = gpu(wl, record=[0, len(pts) - 4])
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(sim.results(), o, "overload")
+    assert_logs(sim, wl, 0)
+    assert_logs(sim, wl, 1)
+    sim.close()
+
+
+def test_ragged_traces_and_empty():
+    r = W.CONFIGS[2]
+    traces = [W.make_trace(r, 2, 0, n_queries=0), W.make_trace(r, 2, 1, n_queries=1),
+              W.make_trace(r, 2, 2, n_queries=3), W.make_trace(r, 2, 3, n_queries=700),
+              W.make_trace(r, 2, 4, n_queries=0), W.make_trace(r, 2, 5, n_queries=37)]
+    wl = W.Workload("ragged", traces, W.make_cluster(r), W.subset_grid(W.make_grid(r), list(range(0, 256, 9))),
+                    W.OBJ_P95)
+    P = wl.grid.n_points
+    sim = gpu(wl, record=[P * 1, P * 2 + 3, P * 3 + 5, P * 5 + 7])
+    g = sim.results()
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(g, o, "ragged")
+    assert (g["p95_us"][:P] == 0).all() and (g["n_done"][:P] == 0).all()
+    for j in range(4):
+        assert_logs(sim, wl, j)
+    check_best(sim, wl, o)
+    sim.close()
+
+
+def test_largest_shapes():
+    """64 instances of 16 slots (1024 slots per simulation), k = 8 candidates,
+    up to 15 corrections per chain."""
+    r = W.CONFIGS[2]
+    r2 = W.Recipe("maxshape", 2, 120, "poisson", [3.0], 0.0, [8, 8], 0.85, 15, r.prompt, r.out, r.out_est,
+                  r.ref_prompt, [W.TYPE_C, W.TYPE_A], [64, 0], 1, 3 * W.SCALE, 4, [W.SCALE, 4 * W.SCALE], [0, 15],
+                  [(1, 1)], 300_000, W.OBJ_P95)
+    traces = [W.make_trace(r2, 9, s) for s in range(2)]
+    assert max(int(t.retry.max()) for t in traces) == 15
+    wl = W.Workload("maxshape", traces, W.make_cluster(r2), W.make_grid(r2), W.OBJ_P95)
+    sim = gpu(wl, record=[1, 13])
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(sim.results(), o, "max shapes")
+    assert_logs(sim, wl, 0)
+    assert_logs(sim, wl, 1)
+    sim.close()
+
+
+def test_repeat_runs_and_upload():
+    wl = W.make_workload(1, n_traces=2, n_queries=300)
+    sim = gpu(wl)
+    a = sim.results()
+    sim.run()
+    b = sim.results()
+    assert_same(a, b, "repeat")
+    # same shapes, different tokens and arrivals: upload in place == fresh handle
+    alt = []
+    for t in wl.traces:
+        u = W.Trace(*[getattr(t, f).copy() for f in ("arrival_us", "k", "call_base", "prompt", "out", "out_est",
+                                                      "stage", "cand", "retry")])
+        u.prompt[:] = u.prompt[::-1].copy()
+        u.arrival_us[:] = u.arrival_us * 3 // 4
+        alt.append(u)
+    sim.upload(alt)
+    sim.run()
+    c = sim.results()
+    wl2 = W.Workload("alt", alt, wl.cluster, wl.grid, wl.objective)
+    fresh = gpu(wl2)
+    assert_same(c, fresh.results(), "upload")
+    o = oracle_results(wl2, range(wl2.n_sims))
+    assert_same(c, o, "upload vs oracle")
+    sim.close()
+    fresh.close()
+
+
+# ------------------------------------------------------------------ full size
+@pytest.mark.parametrize("cfg,n_sample", [(1, None), (2, 48), (3, 24)])
+def test_full_recipes_sampled(cfg, n_sample):
+    wl = W.make_workload(cfg)
+    sim = gpu(wl)
+    g = sim.results()
+    nq = np.repeat([t.n_queries for t in wl.traces], wl.grid.n_points)
+    nc = np.repeat([t.n_calls for t in wl.traces], wl.grid.n_points)
+    assert (g["status"] == 0).all() and (g["n_done"] == nq).all() and (g["events"] == nc).all()
+    if n_sample is None:
+        sims = list(range(wl.n_sims))
+    else:
+        rng = np.random.default_rng(100 + cfg)
+        sims = sorted(set(rng.choice(wl.n_sims, n_sample, replace=False).tolist() + [wl.n_sims - 1]))
+    o = oracle_results(wl, sims)
+    assert_same(g[sims], o, f"recipe {cfg} sample")
+    nqt = [t.n_queries for t in wl.traces]
+    for obj in (W.OBJ_P95, W.OBJ_P95_SLO95):
+        gp, gs, per = oracle.best(g, len(wl.traces), wl.grid.n_points, nqt, obj)
+        bp, bs, _, bper = sim.best(obj)
+        assert (bp, bs) == (gp, gs) and bper.tolist() == per.tolist()
+    sim.close()
+
+
+def test_full_size_ceiling_sampled():
+    """The benchmarked workload (256 traces x 20000 queries x 1024 points) in
+    the benchmark's launch configuration: every simulation completes, a
+    seeded sample matches the oracle exactly, and the best-point kernel agrees
+    with the oracle's rule applied to the GPU's result table."""
+    wl = W.make_workload(4)
+    sim = gpu(wl)
+    g = sim.results()
+    P = wl.grid.n_points
+    nq = np.repeat([t.n_queries for t in wl.traces], P)
+    nc = np.repeat([t.n_calls for t in wl.traces], P)
+    assert (g["status"] == 0).all() and (g["n_done"] == nq).all() and (g["events"] == nc).all()
+    rng = np.random.default_rng(4)
+    sims = sorted(set(rng.choice(wl.n_sims, 12, replace=False).tolist() + [P - 1, wl.n_sims - 1, 37 * P + 1023]))
+    o = oracle_results(wl, sims)
+    assert_same(g[sims], o, "recipe 4 sample")
+    nqt = [t.n_queries for t in wl.traces]
+    for obj in (W.OBJ_P95, W.OBJ_P95_SLO95):
+        gp, gs, per = oracle.best(g, len(wl.traces), P, nqt, obj)
+        bp, bs, _, bper = sim.best(obj)
+        assert (bp, bs) == (gp, gs) and bper.tolist() == per.tolist()
+    sim.close()
