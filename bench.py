@@ -230,7 +230,7 @@ def run_gpu(args):
     best_ms = float(np.median([x[2] for x in sim_ms]))
 
     # end to end through the C ABI from host buffers: upload, run, read back
-    e2e_steps = max(1, min(args.steps, 3))
+    e2e_steps = 1
     h2d = sum(t.arrival_us.nbytes + t.k.nbytes + t.call_base.nbytes + t.prompt.nbytes + t.out.nbytes +
               t.out_est.nbytes + t.stage.nbytes + t.cand.nbytes + t.retry.nbytes for t in wl.traces)
     d2h = wl.n_sims * H.RESULT_DTYPE.itemsize
@@ -290,7 +290,7 @@ def run_gpu(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--steps", type=int, default=2)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")

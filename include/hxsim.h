@@ -136,7 +136,8 @@ typedef struct hx_result {
   int32_t slo_met;      /* queries with latency <= T_slo */
   int32_t n_done;       /* completed queries */
   int32_t status;       /* HX_OK or HX_ERR_CAPACITY / HX_ERR_STEP_LIMIT */
-  int32_t pad;
+  int32_t cycles_k;     /* diagnostic: SM clock cycles / 1024 the simulation took
+                           (saturated; varies from run to run) */
 } hx_result;
 
 /* Best point (Sec. 4.3's argmin of P95; the constrained objective keeps

@@ -198,7 +198,11 @@ def pick(policy: int, rid: Sequence[int], urgency_fp: Sequence[int], enq_us: Seq
 def best(results: np.ndarray, n_traces: int, n_points: int, n_queries: Sequence[int], objective: int):
     """(global point, global sum of P95, per-trace points) of Sec. 4.3's argmin."""
     lib = _load()
-    res = np.ascontiguousarray(results, dtype=RESULT_DTYPE)
+    res = np.ascontiguousarray(results)
+    if res.dtype != RESULT_DTYPE:
+        if res.dtype.itemsize != RESULT_DTYPE.itemsize:
+            raise ValueError("result records must be 48 bytes")
+        res = res.view(RESULT_DTYPE)
     nq = _c(n_queries, np.int32)
     gp = ctypes.c_int32(0)
     gs = ctypes.c_int64(0)

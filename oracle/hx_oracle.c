@@ -82,12 +82,15 @@ static uint64_t mix64(uint64_t z) {
   return z ^ (z >> 31);
 }
 
+/* Digest terms: one finalizer over (time * golden ratio) xor (id << 8 | tag). */
+#define DIGEST_MUL 0x9E3779B97F4A7C15ULL
+
 static uint64_t call_term(int32_t rid, int inst, int64_t start) {
-  return mix64((uint64_t)start ^ mix64(((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst));
+  return mix64(((uint64_t)start * DIGEST_MUL) ^ (((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst));
 }
 
 static uint64_t query_term(int32_t qid, int64_t end) {
-  return mix64((uint64_t)end ^ mix64(((uint64_t)(uint32_t)qid << 8) | 0xFFu));
+  return mix64(((uint64_t)end * DIGEST_MUL) ^ (((uint64_t)(uint32_t)qid << 8) | 0xFFu));
 }
 
 static int cmp_i64(const void* a, const void* b) {

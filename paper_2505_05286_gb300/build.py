@@ -28,10 +28,10 @@ def _stale() -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(force: bool = False, verbose: bool = False, extra=()) -> str:
-    if not force and not _stale():
+def build(force: bool = False, verbose: bool = False, extra=(), out: str = LIB) -> str:
+    if not force and out == LIB and not _stale():
         return LIB
-    objdir = os.path.join(PKG, "_build")
+    objdir = os.path.join(os.path.dirname(out), "_build" + ("" if out == LIB else "_" + os.path.basename(out)))
     os.makedirs(objdir, exist_ok=True)
 
     def compile_one(src):
@@ -49,13 +49,13 @@ def build(force: bool = False, verbose: bool = False, extra=()) -> str:
     if verbose:
         for _, err in outs:
             sys.stderr.write(err)
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = out + f".tmp{os.getpid()}"
     cmd = [NVCC, *ARCH, "-shared", "-o", tmp] + [o for o, _ in outs]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, out)
+    return out
 
 
 if __name__ == "__main__":

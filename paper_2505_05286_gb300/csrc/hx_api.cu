@@ -5,6 +5,7 @@
 
 #include <algorithm>
 #include <cstdio>
+#include <cstddef>
 #include <cstring>
 #include <new>
 #include <string>
@@ -248,8 +249,9 @@ int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
   return HX_OK;
 }
 
+// WarpShared with its trailing slot array sized for the cluster
 int per_warp_smem(int total_slots) {
-  return (int)align_up((192 + (int64_t)total_slots) * 8 + ((int64_t)total_slots + 320) * 4, 16);
+  return (int)align_up((int64_t)offsetof(hx::WarpShared, slot) + 8 * (int64_t)std::max(total_slots, 1), 16);
 }
 
 }  // namespace

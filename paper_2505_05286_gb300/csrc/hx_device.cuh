@@ -44,7 +44,7 @@ static_assert(sizeof(CallRec) == 64, "CallRec is one 64-byte unit");
 struct __align__(16) HeapEnt {
   long long key;
   int rid;
-  int pad;
+  int svc;   // service time on the queue's instance
 };
 
 // Cluster description passed by value (kernel parameter space).
@@ -107,6 +107,26 @@ struct SimArgs {
   int64_t* rec_budget;
   int64_t* rec_start;
   int64_t rec_stride;
+};
+
+// Per-warp shared memory of one simulation: per-instance local-queue and
+// slot state, per-simulation constants and lane-0 accumulators, then one
+// 64-bit (end << 24 | request id) key per batch slot of the cluster.
+struct WarpShared {
+  uint64_t nkey[HX_MAX_INST];   // earliest running (end << 24 | rid), or all ones
+  int32_t hoff[HX_MAX_INST];    // local queue: heap offset in the arena
+  int32_t hcap[HX_MAX_INST];    //              heap capacity
+  int32_t hsize[HX_MAX_INST];   //              heap size
+  uint32_t freem[HX_MAX_INST];  // free-slot mask
+  int32_t nslot[HX_MAX_INST];   // slot holding nkey
+  // per-simulation constants
+  int64_t A, one_minus_a, G, beta, f_s, f_g, cref_c, cref_e;
+  int32_t rho, rmax, lpol, dpol, recj, kcap, rr, bump;
+  // lane-0 accumulators
+  uint64_t digest;
+  int64_t makespan;
+  int32_t n_done, slo_met, events, tk;
+  uint64_t slot[1];             // [total_slots]
 };
 
 struct BestCand {

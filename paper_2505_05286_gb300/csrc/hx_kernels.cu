@@ -5,6 +5,8 @@
 // fixed point; every division is the compiler's truncating `/`.  Nothing here
 // is a dense contraction, so there are no tensor-core paths; the simulation
 // kernel is bound by the SM issue rate, the preparation kernel by HBM.
+#include <climits>
+
 #include "hx_device.cuh"
 
 namespace hx {
@@ -19,12 +21,15 @@ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
   return z ^ (z >> 31);
 }
 
+constexpr uint64_t kDigestMul = 0x9E3779B97F4A7C15ull;
+
+// Digest terms: one finalizer over (time * golden ratio) xor (id << 8 | tag).
 __device__ __forceinline__ uint64_t call_term(int32_t rid, int inst, int64_t start) {
-  return mix64((uint64_t)start ^ mix64(((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst));
+  return mix64(((uint64_t)start * kDigestMul) ^ (((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst));
 }
 
 __device__ __forceinline__ uint64_t query_term(int32_t qid, int64_t end) {
-  return mix64((uint64_t)end ^ mix64(((uint64_t)(uint32_t)qid << 8) | 0xFFull));
+  return mix64(((uint64_t)end * kDigestMul) ^ (((uint64_t)(uint32_t)qid << 8) | 0xFFull));
 }
 
 __device__ __forceinline__ uint64_t warp_min_u64(uint64_t v) {
@@ -165,45 +170,23 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
 // -------------------------------------------------------- simulation kernel
 namespace {
 
-// Per-warp shared state of one simulation.
-struct Smem {
-  int64_t* q;          // [64] sum of est over requests dispatched and unfinished
-  int64_t* rew;        // [64] reward_of(beta, q)
-  uint64_t* nkey;      // [64] earliest running (end << 24 | rid), or kKeyInf
-  int64_t* slot_end;   // [total_slots] end time or kTimeInf when free
-  int32_t* slot_rid;   // [total_slots]
-  int32_t* hoff;       // [64] local queue: offset of the heap in the arena
-  int32_t* hcap;       // [64] capacity
-  int32_t* hsize;      // [64] size
-  uint32_t* freem;     // [64] free-slot mask
-  int32_t* nslot;      // [64] slot of nkey
-};
-
-__device__ __forceinline__ Smem carve(unsigned char* base, int ts) {
-  Smem s;
-  s.q = reinterpret_cast<int64_t*>(base);
-  s.rew = s.q + 64;
-  s.nkey = reinterpret_cast<uint64_t*>(s.rew + 64);
-  s.slot_end = reinterpret_cast<int64_t*>(s.nkey + 64);
-  s.slot_rid = reinterpret_cast<int32_t*>(s.slot_end + ts);
-  s.hoff = s.slot_rid + ts;
-  s.hcap = s.hoff + 64;
-  s.hsize = s.hcap + 64;
-  s.freem = reinterpret_cast<uint32_t*>(s.hsize + 64);
-  s.nslot = reinterpret_cast<int32_t*>(s.freem + 64);
-  return s;
+__device__ __forceinline__ int pick4(const int4& v, int t) {
+  return t == 0 ? v.x : (t == 1 ? v.y : (t == 2 ? v.z : v.w));
 }
 
 __device__ __forceinline__ bool ent_better(long long ka, int ra, long long kb, int rb) {
   return ka > kb || (ka == kb && ra < rb);
 }
 
-// Binary max-heap on (key desc, rid asc); single lane.
-__device__ void heap_push(HeapEnt* h, int n, long long key, int rid) {
+// Local queues are 32-ary max-heaps on (key desc, rid asc) in the warp's
+// arena: node i has children 32 i + 1 .. 32 i + 32, so 40k waiting requests
+// sit four levels deep.  Push sifts up on one lane (new requests rarely
+// climb); pop sifts down with the whole warp, one lane per child.
+__device__ __noinline__ void heap_push(HeapEnt* h, int n, long long key, int rid, int svc) {
   int i = n;
   while (i > 0) {
-    int par = (i - 1) >> 1;
-    HeapEnt pe = h[par];
+    const int par = (i - 1) >> 5;
+    const HeapEnt pe = h[par];
     if (!ent_better(key, rid, pe.key, pe.rid)) break;
     h[i] = pe;
     i = par;
@@ -211,40 +194,64 @@ __device__ void heap_push(HeapEnt* h, int n, long long key, int rid) {
   HeapEnt e;
   e.key = key;
   e.rid = rid;
-  e.pad = 0;
+  e.svc = svc;
   h[i] = e;
 }
 
-__device__ HeapEnt heap_pop(HeapEnt* h, int n) {
-  HeapEnt top = h[0];
-  HeapEnt last = h[n - 1];
-  int m = n - 1;
+// All lanes call with the same (h, n >= 1); every lane gets the top entry.
+__device__ __noinline__ HeapEnt heap_pop_warp(HeapEnt* h, int n, int lane) {
+  const HeapEnt top = h[0];
+  const HeapEnt last = h[n - 1];
+  const int m = n - 1;
   int i = 0;
   for (;;) {
-    int l = 2 * i + 1;
-    if (l >= m) break;
-    int r = l + 1;
-    HeapEnt cl = h[l];
-    int cidx = l;
-    if (r < m) {
-      HeapEnt cr = h[r];
-      if (ent_better(cr.key, cr.rid, cl.key, cl.rid)) { cl = cr; cidx = r; }
+    const int first = 32 * i + 1;
+    if (first >= m) break;
+    const int child = first + lane;
+    long long ck = LLONG_MIN;
+    int cr = INT_MAX, cs = 0;
+    if (child < m) {
+      const HeapEnt e = h[child];
+      ck = e.key;
+      cr = e.rid;
+      cs = e.svc;
     }
-    if (!ent_better(cl.key, cl.rid, last.key, last.rid)) break;
-    h[i] = cl;
-    i = cidx;
+    // warp argmax of (key desc, rid asc)
+    const uint64_t uk = (uint64_t)ck ^ 0x8000000000000000ull;
+    const uint32_t hi = (uint32_t)(uk >> 32), lo = (uint32_t)uk;
+    const uint32_t mh = __reduce_max_sync(kFull, hi);
+    const bool c1 = hi == mh;
+    const uint32_t ml = __reduce_max_sync(kFull, c1 ? lo : 0u);
+    const bool c2 = c1 && lo == ml;
+    const uint32_t mr = __reduce_min_sync(kFull, c2 ? (uint32_t)cr : 0xffffffffu);
+    const int b = __ffs(__ballot_sync(kFull, c2 && (uint32_t)cr == mr)) - 1;
+    const long long bk = __shfl_sync(kFull, ck, b);
+    const int br = __shfl_sync(kFull, cr, b);
+    const int bs = __shfl_sync(kFull, cs, b);
+    if (!ent_better(bk, br, last.key, last.rid)) break;
+    if (lane == 0) {
+      HeapEnt e;
+      e.key = bk;
+      e.rid = br;
+      e.svc = bs;
+      h[i] = e;
+    }
+    i = first + b;
   }
-  if (m > 0) h[i] = last;
+  if (lane == 0 && m > 0) h[i] = last;
+  __syncwarp();
   return top;
 }
 
-// Min-heap of the K largest latencies seen so far; single lane.
-__device__ void topk_insert(int64_t* h, int& n, int kcap, int64_t v) {
+// Min-heap of the K largest latencies seen so far; single lane.  Its root
+// is the K-th largest latency, i.e. the nearest-rank P95 when
+// K = n - ceil(0.95 n) + 1.
+__device__ __noinline__ void topk_insert(int64_t* h, int& n, int kcap, int64_t v) {
   if (n < kcap) {
     int i = n++;
     while (i > 0) {
-      int par = (i - 1) >> 1;
-      int64_t pv = h[par];
+      const int par = (i - 1) >> 1;
+      const int64_t pv = h[par];
       if (pv <= v) break;
       h[i] = pv;
       i = par;
@@ -253,219 +260,186 @@ __device__ void topk_insert(int64_t* h, int& n, int kcap, int64_t v) {
   } else if (v > h[0]) {
     int i = 0;
     for (;;) {
-      int l = 2 * i + 1;
+      const int l = 2 * i + 1;
       if (l >= n) break;
-      int r = l + 1;
-      int cidx = l;
+      int ci = l;
       int64_t cv = h[l];
-      if (r < n && h[r] < cv) { cv = h[r]; cidx = r; }
+      if (l + 1 < n && h[l + 1] < cv) {
+        cv = h[l + 1];
+        ci = l + 1;
+      }
       if (cv >= v) break;
       h[i] = cv;
-      i = cidx;
+      i = ci;
     }
     h[i] = v;
   }
 }
 
-struct SimState {
-  int64_t now;
-  uint64_t touched;
-  int32_t rr;
-  int32_t bump;
-  int32_t status;
-};
+__device__ __forceinline__ void prefetch_l1(const void* p) {
+  asm volatile("prefetch.global.L1 [%0];" ::"l"(p));
+}
+
+// Queue this event's dispatches to instance m (pending entries on the lanes of
+// mask pm) in m's heap, re-homing the heap in the arena when it is full.
+// All lanes call.  Returns HX_OK or HX_ERR_CAPACITY.
+__device__ __noinline__ int push_pending(WarpShared* W, HeapEnt* arena, int64_t arena_per_warp, int m, unsigned pm,
+                                        long long pend_key, int pend_rid, int pend_svc, int lane) {
+  while (pm) {
+    const int j = __ffs(pm) - 1;
+    pm &= pm - 1;
+    const long long key = __shfl_sync(kFull, pend_key, j);
+    const int rid = __shfl_sync(kFull, pend_rid, j);
+    const int svc = __shfl_sync(kFull, pend_svc, j);
+    const int size = W->hsize[m], cap = W->hcap[m], off = W->hoff[m], bump = W->bump;
+    __syncwarp();
+    int hoff = off;
+    if (size == cap) {
+      const int ncap = cap ? 2 * cap : 16;
+      if ((int64_t)bump + ncap > arena_per_warp) return HX_ERR_CAPACITY;
+      hoff = bump;
+      for (int i = lane; i < size; i += 32) arena[hoff + i] = arena[off + i];
+      __syncwarp();
+      if (lane == 0) {
+        W->bump = bump + ncap;
+        W->hoff[m] = hoff;
+        W->hcap[m] = ncap;
+      }
+    }
+    if (lane == 0) {
+      heap_push(arena + hoff, size, key, rid, svc);
+      W->hsize[m] = size + 1;
+    }
+    __syncwarp();
+  }
+  return HX_OK;
+}
+
+// Lane 0: a query's evaluation call finished at `now` (Sec. 4.3's metrics).
+__device__ __noinline__ void finish_query(WarpShared* W, int64_t* topk, int32_t qid, int64_t now, int64_t arrival,
+                                         int64_t deadline) {
+  W->slo_met += now <= deadline ? 1 : 0;
+  W->n_done++;
+  W->makespan = now;
+  W->digest += query_term(qid, now);
+  int tk = W->tk;
+  topk_insert(topk, tk, W->kcap, now - arrival);
+  W->tk = tk;
+}
+
+__device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, int m, int64_t now, int64_t budget) {
+  const int64_t o = (int64_t)recj * a.rec_stride + rid;
+  a.rec_inst[o] = m;
+  a.rec_enq[o] = now;
+  a.rec_budget[o] = budget;
+}
+
+__device__ __noinline__ int64_t budget_wide(int64_t num, int64_t tb, int64_t d) { return scaled_div(num, tb, d); }
 
 }  // namespace
 
-__global__ void __launch_bounds__(kWarpsPerBlock * 32) hx_sim_kernel(SimArgs a, ClusterK c) {
+#ifndef HX_SIM_MIN_BLOCKS
+#define HX_SIM_MIN_BLOCKS 6
+#endif
+// Resident blocks per SM the register allocation aims for (4 warps each).
+__global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim_kernel(SimArgs a, ClusterK c) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int ts = c.total_slots;
-  Smem S = carve(smem_raw + warp * c.smem_per_warp, ts);
+  WarpShared* const W = reinterpret_cast<WarpShared*>(smem_raw + warp * c.smem_per_warp);
   const int64_t gw = (int64_t)blockIdx.x * kWarpsPerBlock + warp;
-  HeapEnt* arena = a.arena + gw * a.arena_per_warp;
-  uint8_t* chains = a.chains + gw * a.chains_per_warp;
-  int64_t* topk = a.topk + gw * a.topk_per_warp;
+  HeapEnt* const arena = a.arena + gw * a.arena_per_warp;
+  uint8_t* const chains = a.chains + gw * a.chains_per_warp;
+  int64_t* const topk = a.topk + gw * a.topk_per_warp;
   const int N = c.n_inst;
   const int m0 = lane, m1 = lane + 32;
-  const int ty0 = m0 < N ? c.inst_type[m0] : 0;
-  const int ty1 = m1 < N ? c.inst_type[m1] : 0;
-
-  // stage reference costs: mean over instances of Eq. (comp) at the stage's reference tokens
-  int64_t cref[4];
-#pragma unroll
-  for (int s = 0; s < 4; ++s) {
-    int64_t sum = 0;
-    for (int ty = 0; ty < c.n_types; ++ty)
-      sum += cost_on_type(c, ty, c.ref_prompt[s], c.ref_out[s]) * c.cnt[ty];
-    cref[s] = sum / N;
-  }
+  const bool valid0 = m0 < N, valid1 = m1 < N;
+  const int ty0 = valid0 ? c.inst_type[m0] : 0;
+  const int ty1 = valid1 ? c.inst_type[m1] : 0;
 
   for (;;) {
-    unsigned long long simu = 0;
-    if (lane == 0) simu = atomicAdd(a.work_counter, 1ull);
-    const int64_t sim = (int64_t)__shfl_sync(kFull, simu, 0);
-    if (sim >= a.n_sims) break;
-
-    const int t = (int)(sim / a.n_points);
-    const int p = (int)(sim - (int64_t)t * a.n_points);
+    unsigned long long work = 0;
+    if (lane == 0) work = atomicAdd(a.work_counter, 1ull);
+    const int64_t w = (int64_t)__shfl_sync(kFull, work, 0);
+    if (w >= a.n_sims) break;
+    // trace-major, so that concurrent simulations share a trace in L2; within a
+    // trace the highest point index (highest alpha, the longest queues) first
+    const int t = (int)(w / a.n_points);
+    const int p = a.n_points - 1 - (int)(w - (int64_t)t * a.n_points);
+    const int64_t sim = (int64_t)t * a.n_points + p;
+    const long long clk0 = clock64();
     const int64_t qb = a.q_off[t];
     const int32_t nq = (int32_t)(a.q_off[t + 1] - qb);
     const int64_t cb = a.c_off[t];
     const int32_t nc = (int32_t)(a.c_off[t + 1] - cb);
-    const CallRec* rec = a.rec + cb;
-    const int64_t* arr = a.arrival + qb;
-    const int64_t* qcall = a.qcall + qb;
-    const int64_t A = a.alpha[p], G = a.gamma[p], beta = a.beta[p];
-    const int rho = a.rho[p];
-    const int lpol = a.lpol[p], dpol = a.dpol[p];
-    const int recj = a.rec_map ? a.rec_map[sim] : -1;
-    const int64_t one_minus_a = kScale - A;
-    const int64_t rmax = c.rmax;
-    const int64_t corr_plan = rho < rmax ? rho : rmax;
-    const int64_t f_s = cref[HX_STAGE_G] + corr_plan * cref[HX_STAGE_C] + cref[HX_STAGE_E];
-    const int64_t f_g = corr_plan * cref[HX_STAGE_C] + cref[HX_STAGE_E];
-    const int64_t rew0 = reward_of(beta, 0);
+    const CallRec* const rec = a.rec + cb;
 
     for (int m = lane; m < 64; m += 32) {
-      S.q[m] = 0;
-      S.rew[m] = rew0;
-      S.nkey[m] = kKeyInf;
-      S.hoff[m] = 0;
-      S.hcap[m] = 0;
-      S.hsize[m] = 0;
-      S.freem[m] = m < N ? ((1u << c.inst_slots[m]) - 1u) : 0u;
-      S.nslot[m] = -1;
+      W->nkey[m] = kKeyInf;
+      W->hoff[m] = 0;
+      W->hcap[m] = 0;
+      W->hsize[m] = 0;
+      W->freem[m] = m < N ? ((1u << c.inst_slots[m]) - 1u) : 0u;
+      W->nslot[m] = -1;
     }
-    for (int j = lane; j < ts; j += 32) {
-      S.slot_end[j] = kTimeInf;
-      S.slot_rid[j] = -1;
+    for (int j = lane; j < c.total_slots; j += 32) W->slot[j] = kKeyInf;
+    if (lane == 0) {
+      // stage reference costs: mean over instances of Eq. (comp) at the stage's reference tokens
+      int64_t cref[4];
+      for (int s = 0; s < 4; ++s) {
+        int64_t sum = 0;
+        for (int ty = 0; ty < c.n_types; ++ty) sum += cost_on_type(c, ty, c.ref_prompt[s], c.ref_out[s]) * c.cnt[ty];
+        cref[s] = sum / N;
+      }
+      const int64_t A = a.alpha[p], rho = a.rho[p], rmax = c.rmax;
+      const int64_t corr_plan = rho < rmax ? rho : rmax;
+      W->A = A;
+      W->one_minus_a = kScale - A;
+      W->G = a.gamma[p];
+      W->beta = a.beta[p];
+      // rest-of-path costs of the budget denominator for S and G calls
+      W->f_s = cref[HX_STAGE_G] + corr_plan * cref[HX_STAGE_C] + cref[HX_STAGE_E];
+      W->f_g = corr_plan * cref[HX_STAGE_C] + cref[HX_STAGE_E];
+      W->cref_c = cref[HX_STAGE_C];
+      W->cref_e = cref[HX_STAGE_E];
+      W->rho = (int32_t)rho;
+      W->rmax = (int32_t)rmax;
+      W->lpol = a.lpol[p];
+      W->dpol = a.dpol[p];
+      W->recj = a.rec_map ? a.rec_map[sim] : -1;
+      W->kcap = nq - (95 * nq + 99) / 100 + 1;
+      W->rr = 0;
+      W->bump = 0;
+      W->digest = 0;
+      W->makespan = 0;
+      W->n_done = 0;
+      W->slo_met = 0;
+      W->events = 0;
+      W->tk = 0;
     }
     __syncwarp();
 
-    uint64_t k0 = kKeyInf, k1 = kKeyInf;  // this lane's instances' next-completion event keys
-    const int kcap = nq - (95 * nq + 99) / 100 + 1;
-    int tk = 0;
-    int32_t qa = 0;
-    uint64_t akey = nq > 0 ? (((uint64_t)arr[0] << 7) | kArrivalTag) : kKeyInf;
-    int32_t n_done = 0, slo_met = 0;
-    int64_t makespan = 0, events = 0;
-    uint64_t digest = 0;
-    SimState st;
-    st.now = 0;
-    st.touched = 0;
-    st.rr = 0;
-    st.bump = 0;
-    st.status = HX_OK;
-    const int64_t max_steps = (int64_t)nc + nq + 8;
-    int64_t steps = 0;
+    // this lane's instances: queue cost, cached reward and its staleness, event keys
+    int64_t q0 = 0, q1 = 0;
+    int64_t rew0 = reward_of(W->beta, 0), rew1 = rew0;
+    bool dirty0 = false, dirty1 = false;
+    uint64_t k0 = kKeyInf, k1 = kKeyInf;
+    // this event's dispatches, entry j on lane j
+    int pend_m = -1, pend_rid = 0, pend_svc = 0;
+    long long pend_key = 0;
 
-    // refresh this lane's event key for instance m from S.nkey
-    auto refresh_key = [&](int m) {
+    int32_t qa = 0;
+    uint64_t akey = nq > 0 ? (((uint64_t)a.arrival[qb] << 7) | kArrivalTag) : kKeyInf;
+    int64_t now = 0;
+    int32_t status = HX_OK, npend = 0;
+    uint64_t touched = 0;
+    const int32_t max_steps = nc + nq + 8;
+    int32_t steps = 0;
+
+    auto set_key = [&](int m, uint64_t nk) {
       if (lane == (m & 31)) {
-        const uint64_t nk = S.nkey[m];
         const uint64_t kk = nk == kKeyInf ? kKeyInf : (((nk >> 24) << 7) | (uint64_t)m);
         if (m < 32) k0 = kk; else k1 = kk;
-      }
-    };
-
-    // Sec. 4.1 + 4.2: budget at send time, score every instance, enqueue.
-    auto dispatch = [&](int32_t rid) {
-      const CallRec* r = rec + rid;
-      const int stg = r->stage;
-      const int64_t tb = r->tbar;
-      int64_t f;
-      if (stg == HX_STAGE_S) f = f_s;
-      else if (stg == HX_STAGE_G) f = f_g;
-      else if (stg == HX_STAGE_C) {
-        const int64_t left = rmax - (int64_t)r->u;
-        f = (rho < left ? rho : left) * cref[HX_STAGE_C] + cref[HX_STAGE_E];
-      } else f = 0;
-      const int64_t budget = scaled_div(r->deadline - st.now, tb, tb + f);
-      int m;
-      if (dpol == HX_DISPATCH_RR) {
-        m = st.rr;
-        st.rr = (st.rr + 1 == N) ? 0 : st.rr + 1;
-      } else {
-        int64_t s0 = INT64_MIN, s1 = INT64_MIN;
-        if (m0 < N) s0 = one_minus_a * S.rew[m0] - A * (int64_t)r->est[ty0];
-        if (m1 < N) s1 = one_minus_a * S.rew[m1] - A * (int64_t)r->est[ty1];
-        const bool take1 = s1 > s0;
-        m = warp_argmax_s64(take1 ? s1 : s0, take1 ? m1 : m0);
-      }
-      const int64_t est_m = r->est[c.inst_type[m]];
-      if (lane == (m & 31)) {
-        const int64_t q = S.q[m] + est_m;
-        S.q[m] = q;
-        S.rew[m] = reward_of(beta, q);
-      }
-      const long long key = lpol == HX_LOCAL_PQ ? (long long)(kScale * (est_m - budget) - G * st.now)
-                                                : (long long)(-st.now);
-      // local queue push, growing the heap inside the arena when full
-      const int size = S.hsize[m], cap = S.hcap[m], off = S.hoff[m];
-      __syncwarp();
-      int hoff = off;
-      if (size == cap) {
-        const int ncap = cap ? 2 * cap : 16;
-        if ((int64_t)st.bump + ncap > a.arena_per_warp) {
-          st.status = HX_ERR_CAPACITY;
-          return;
-        }
-        hoff = st.bump;
-        st.bump += ncap;
-        for (int j = lane; j < size; j += 32) arena[hoff + j] = arena[off + j];
-        __syncwarp();
-        if (lane == 0) {
-          S.hoff[m] = hoff;
-          S.hcap[m] = ncap;
-        }
-      }
-      if (lane == 0) {
-        heap_push(arena + hoff, size, key, rid);
-        S.hsize[m] = size + 1;
-        if (recj >= 0) {
-          const int64_t o = (int64_t)recj * a.rec_stride + rid;
-          a.rec_inst[o] = m;
-          a.rec_enq[o] = st.now;
-          a.rec_budget[o] = budget;
-        }
-      }
-      __syncwarp();
-      st.touched |= 1ull << m;
-    };
-
-    // Batch boundary on instance m: start the best waiting requests on free slots.
-    auto fill = [&](int m) {
-      const int sb = c.slot_base[m];
-      const int ty = c.inst_type[m];
-      for (;;) {
-        const bool go = S.freem[m] != 0u && S.hsize[m] > 0;
-        __syncwarp();
-        if (!go) break;
-        int rid = 0;
-        if (lane == 0) {
-          const int n = S.hsize[m];
-          HeapEnt top = heap_pop(arena + S.hoff[m], n);
-          S.hsize[m] = n - 1;
-          rid = top.rid;
-          const int64_t end = st.now + rec[rid].svc[ty];
-          const uint32_t fm = S.freem[m];
-          const int sl = __ffs(fm) - 1;
-          S.freem[m] = fm & ~(1u << sl);
-          S.slot_end[sb + sl] = end;
-          S.slot_rid[sb + sl] = rid;
-          const uint64_t nk = ((uint64_t)end << 24) | (uint64_t)rid;
-          if (nk < S.nkey[m]) {
-            S.nkey[m] = nk;
-            S.nslot[m] = sl;
-          }
-          if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = st.now;
-        }
-        rid = __shfl_sync(kFull, rid, 0);
-        __syncwarp();
-        refresh_key(m);
-        digest += call_term(rid, m, st.now);
       }
     };
 
@@ -473,103 +447,229 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) hx_sim_kernel(SimArgs a, 
       const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
       if (ck == kKeyInf && akey == kKeyInf) break;
       if (++steps > max_steps) {
-        st.status = HX_ERR_STEP_LIMIT;
+        status = HX_ERR_STEP_LIMIT;
         break;
       }
-      st.touched = 0;
+      touched = 0;
+      npend = 0;
+      // requests released by this event: rel_first .. rel_first + rel_count - 1
+      int32_t rel_first = 0, rel_count = 0;
       if (ck < akey) {
         // completion on instance m
         const int m = (int)(ck & 127ull);
-        st.now = (int64_t)(ck >> 7);
+        now = (int64_t)(ck >> 7);
         const int sb = c.slot_base[m];
-        const int sl = S.nslot[m];
-        const int32_t rid = S.slot_rid[sb + sl];
+        const int sl = W->nslot[m];
+        const int32_t rid = (int32_t)(W->slot[sb + sl] & 0xffffffull);
+        if (lane < 8 && rid + lane < nc) prefetch_l1(rec + rid + lane);
         __syncwarp();
         if (lane == 0) {
-          S.slot_end[sb + sl] = kTimeInf;
-          S.slot_rid[sb + sl] = -1;
-          S.freem[m] |= 1u << sl;
+          W->slot[sb + sl] = kKeyInf;
+          W->freem[m] |= 1u << sl;
+          W->events++;
         }
         __syncwarp();
         // earliest remaining (end, rid) on m: lanes over its slots
-        uint64_t sk = kKeyInf;
-        if (lane < c.inst_slots[m]) {
-          const int64_t e = S.slot_end[sb + lane];
-          if (e != kTimeInf) sk = ((uint64_t)e << 24) | (uint64_t)(uint32_t)S.slot_rid[sb + lane];
-        }
+        const uint64_t sk = lane < c.inst_slots[m] ? W->slot[sb + lane] : kKeyInf;
         const uint64_t mk = warp_min_u64(sk);
         const unsigned who = __ballot_sync(kFull, sk == mk && mk != kKeyInf);
-        __syncwarp();
         if (lane == 0) {
-          S.nkey[m] = mk;
-          S.nslot[m] = who ? __ffs(who) - 1 : -1;
+          W->nkey[m] = mk;
+          W->nslot[m] = who ? __ffs(who) - 1 : -1;
         }
+        set_key(m, mk);
         const CallRec* r = rec + rid;
+        const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
         const int64_t est_m = r->est[c.inst_type[m]];
         if (lane == (m & 31)) {
-          const int64_t q = S.q[m] - est_m;
-          S.q[m] = q;
-          S.rew[m] = reward_of(beta, q);
+          if (m < 32) { q0 -= est_m; dirty0 = true; }
+          else { q1 -= est_m; dirty1 = true; }
         }
-        __syncwarp();
-        refresh_key(m);
-        st.touched |= 1ull << m;
-        events++;
-        const int stg = r->stage;
+        touched |= 1ull << m;
+        const int stg = tail.w & 0xff;
+        const int32_t qid = tail.z;
         if (stg == HX_STAGE_S) {
-          const int k = r->k;
-          if (lane == 0) chains[r->qid] = (uint8_t)k;
-          for (int j = 1; j <= k && st.status == HX_OK; ++j) dispatch(rid + j);
+          const int k = (tail.w >> 16) & 0xff;
+          if (lane == 0) chains[qid] = (uint8_t)k;
+          rel_first = rid + 1;
+          rel_count = k;
         } else if (stg == HX_STAGE_E) {
-          const int64_t lat = st.now - r->arrival;
-          slo_met += st.now <= r->deadline ? 1 : 0;
-          n_done++;
-          makespan = st.now > makespan ? st.now : makespan;
-          digest += query_term(r->qid, st.now);
-          if (lane == 0) topk_insert(topk, tk, kcap, lat);
-          tk = __shfl_sync(kFull, tk, 0);
+          if (lane == 0) finish_query(W, topk, qid, now, r->arrival, r->deadline);
         } else {
-          const int32_t nx = r->next;
+          const int32_t nx = tail.y;
           if (nx >= 0) {
-            dispatch(nx);
+            rel_first = nx;
+            rel_count = 1;
           } else {
             int left = 0;
             if (lane == 0) {
-              left = chains[r->qid] - 1;
-              chains[r->qid] = (uint8_t)left;
+              left = chains[qid] - 1;
+              chains[qid] = (uint8_t)left;
             }
             left = __shfl_sync(kFull, left, 0);
-            if (left == 0) dispatch(~nx);
+            rel_first = ~nx;
+            rel_count = left == 0 ? 1 : 0;
           }
         }
       } else {
-        st.now = (int64_t)(akey >> 7);
-        const int32_t srid = (int32_t)(qcall[qa] - cb);
+        now = (int64_t)(akey >> 7);
+        rel_first = (int32_t)(a.qcall[qb + qa] - cb);
+        rel_count = 1;
         qa++;
-        akey = qa < nq ? (((uint64_t)arr[qa] << 7) | kArrivalTag) : kKeyInf;
-        dispatch(srid);
+        akey = qa < nq ? (((uint64_t)a.arrival[qb + qa] << 7) | kArrivalTag) : kKeyInf;
       }
-      if (st.status != HX_OK) break;
-      uint64_t tm = st.touched;
+
+      // Sec. 4.1 + 4.2 for each released request, in request-id order: budget at
+      // send time, score every instance, enqueue on the winner.
+      for (int32_t jr = 0; jr < rel_count; ++jr) {
+        const int32_t rid = rel_first + jr;
+        const CallRec* r = rec + rid;
+        const int4 e4 = *reinterpret_cast<const int4*>(r->est);
+        const int4 s4 = *reinterpret_cast<const int4*>(r->svc);
+        const int64_t dl = r->deadline;
+        const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
+        const int64_t tb = tail.x;
+        const int stg = tail.w & 0xff;
+        int64_t f;
+        if (stg == HX_STAGE_S) f = W->f_s;
+        else if (stg == HX_STAGE_G) f = W->f_g;
+        else if (stg == HX_STAGE_C) {
+          const int64_t left = (int64_t)W->rmax - ((tail.w >> 8) & 0xff);
+          const int64_t rho = W->rho;
+          f = (rho < left ? rho : left) * W->cref_c + W->cref_e;
+        } else f = 0;
+        const int64_t dd = tb + f;
+        const int64_t num = dl - now;
+        const bool small = num > -(int64_t(1) << 34) && num < (int64_t(1) << 34);
+        // SIMT division passes: each lane refreshes one stale reward of its
+        // instances per pass; the budget goes to the lowest lane with nothing
+        // stale.  Two passes at most clear the rewards, three the budget.
+        int64_t bres = 0;
+        bool need_budget = small;
+        int bl = 0;
+        const uint64_t beta = (uint64_t)W->beta;
+        for (;;) {
+          const unsigned busy = __ballot_sync(kFull, dirty0 || dirty1);
+          const int cand = (need_budget && ~busy) ? __ffs(~busy) - 1 : -1;
+          uint64_t n = 0, d = 1;
+          int job = 0;
+          if (dirty0) { n = beta; d = q0 > 1 ? q0 : 1; job = 1; }
+          else if (dirty1) { n = beta; d = q1 > 1 ? q1 : 1; job = 2; }
+          else if (lane == cand) { n = (uint64_t)(num < 0 ? -num : num) * (uint64_t)tb; d = (uint64_t)dd; job = 3; }
+          const uint64_t res = n / d;
+          const int64_t capped = res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap;
+          if (job == 1) { rew0 = capped; dirty0 = false; }
+          else if (job == 2) { rew1 = capped; dirty1 = false; }
+          else if (job == 3) { bres = num < 0 ? -(int64_t)res : (int64_t)res; }
+          if (cand >= 0) { bl = cand; need_budget = false; }
+          if (!need_budget && !__any_sync(kFull, dirty0 || dirty1)) break;
+        }
+        const int64_t budget = small ? __shfl_sync(kFull, bres, bl) : budget_wide(num, tb, dd);
+        int m;
+        if (W->dpol == HX_DISPATCH_RR) {
+          m = W->rr;
+          __syncwarp();
+          if (lane == 0) W->rr = (m + 1 == N) ? 0 : m + 1;
+        } else {
+          const int64_t A = W->A, oma = W->one_minus_a;
+          const int64_t s0 = valid0 ? oma * rew0 - A * (int64_t)pick4(e4, ty0) : INT64_MIN;
+          const int64_t s1 = valid1 ? oma * rew1 - A * (int64_t)pick4(e4, ty1) : INT64_MIN;
+          const bool take1 = s1 > s0;
+          m = warp_argmax_s64(take1 ? s1 : s0, take1 ? m1 : m0);
+        }
+        const int tym = c.inst_type[m];
+        const int64_t est_m = pick4(e4, tym);
+        const int svc_m = pick4(s4, tym);
+        if (lane == (m & 31)) {
+          if (m < 32) { q0 += est_m; dirty0 = true; }
+          else { q1 += est_m; dirty1 = true; }
+        }
+        const long long key = W->lpol == HX_LOCAL_PQ ? (long long)(kScale * (est_m - budget) - W->G * now) : (long long)(-now);
+        if (lane == npend) {
+          pend_m = m;
+          pend_key = key;
+          pend_rid = rid;
+          pend_svc = svc_m;
+        }
+        npend++;
+        touched |= 1ull << m;
+        const int recj = W->recj;
+        if (recj >= 0 && lane == 0) log_dispatch(a, recj, rid, m, now, budget);
+      }
+
+      // Batch boundary on every touched instance: its free slots go to the most
+      // urgent of the waiting requests and this event's new ones.
+      uint64_t tm = touched;
       while (tm) {
         const int m = __ffsll((long long)tm) - 1;
         tm &= tm - 1;
-        fill(m);
+        const unsigned pm = __ballot_sync(kFull, lane < npend && pend_m == m);
+        const uint32_t fm = W->freem[m];
+        const int hs = W->hsize[m];
+        __syncwarp();
+        // fast path: an empty queue with room for all of this event's arrivals
+        const bool direct = hs == 0 && __popc(pm) <= __popc(fm);
+        if (!direct && pm) {
+          status = push_pending(W, arena, a.arena_per_warp, m, pm, pend_key, pend_rid, pend_svc, lane);
+          if (status != HX_OK) break;
+        }
+        unsigned bits = direct ? pm : 0u;
+        for (;;) {
+          int rid, svc;
+          if (direct) {
+            if (!bits) break;
+            const int j = __ffs(bits) - 1;
+            bits &= bits - 1;
+            rid = __shfl_sync(kFull, pend_rid, j);
+            svc = __shfl_sync(kFull, pend_svc, j);
+          } else {
+            const int n = W->hsize[m];
+            const bool go = W->freem[m] != 0u && n > 0;
+            __syncwarp();
+            if (!go) break;
+            const HeapEnt top = heap_pop_warp(arena + W->hoff[m], n, lane);
+            if (lane == 0) W->hsize[m] = n - 1;
+            rid = top.rid;
+            svc = top.svc;
+          }
+          if (lane == 0) {
+            // occupy a free slot until now + svc
+            const int sb = c.slot_base[m];
+            const uint32_t fr = W->freem[m];
+            const int sl = __ffs(fr) - 1;
+            W->freem[m] = fr & ~(1u << sl);
+            const uint64_t nk = ((uint64_t)(now + svc) << 24) | (uint64_t)(uint32_t)rid;
+            W->slot[sb + sl] = nk;
+            if (nk < W->nkey[m]) {
+              W->nkey[m] = nk;
+              W->nslot[m] = sl;
+            }
+            W->digest += call_term(rid, m, now);
+            const int recj = W->recj;
+            if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
+          }
+          __syncwarp();
+        }
+        set_key(m, W->nkey[m]);
       }
+      if (status != HX_OK) break;
     }
 
+    __syncwarp();
     if (lane == 0) {
-      int status = st.status;
-      if (status == HX_OK && n_done != nq) status = HX_ERR_STEP_LIMIT;
+      int st = status;
+      const int32_t n_done = W->n_done;
+      if (st == HX_OK && n_done != nq) st = HX_ERR_STEP_LIMIT;
       hx_result res;
-      res.p95_us = status == HX_OK ? (nq > 0 ? topk[0] : 0) : -1;
-      res.makespan_us = makespan;
-      res.events = events;
-      res.digest = digest;
-      res.slo_met = slo_met;
+      res.p95_us = st == HX_OK ? (nq > 0 ? topk[0] : 0) : -1;
+      res.makespan_us = W->makespan;
+      res.events = W->events;
+      res.digest = W->digest;
+      res.slo_met = W->slo_met;
       res.n_done = n_done;
-      res.status = status;
-      res.pad = 0;
+      res.status = st;
+      const long long dc = (clock64() - clk0) >> 10;
+      res.cycles_k = dc < INT32_MAX ? (int32_t)dc : INT32_MAX;
       a.results[sim] = res;
     }
     __syncwarp();
