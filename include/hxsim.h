@@ -192,6 +192,35 @@ int hx_sim_prep(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int3
  * opt.timing = 1.  Waits for the run. */
 int hx_sim_timings(hx_sim* h, float* prep_ms, float* sim_ms, float* best_ms);
 
+/* Size of the device array behind hx_sim_run_static. */
+#define HX_STATIC_SCRATCH_BYTES (64u << 20)
+
+/* The whole path (preparation, every simulation of one trace, best point)
+ * without allocating any memory, for callers that cannot allocate device
+ * memory: code that runs where cudaMalloc is not allowed or not available (a
+ * plugin or service whose host process owns every allocation, a real-time
+ * loop that must not enter the allocator), or that cannot keep a handle.
+ * It has no counterpart in the paper.
+ *
+ * Inputs (one trace, the cluster, the grid) and outputs (`results`, host
+ * [n_points], and optionally `best` for `objective`) are the caller's host
+ * memory, validated exactly as hx_sim_create validates them.  Every
+ * intermediate buffer -- the copied inputs, the per-call records, the
+ * per-warp local-queue arenas, the results -- is carved from one file-scope
+ * device array of HX_STATIC_SCRATCH_BYTES (64 MiB), which every GPU that
+ * loads the library holds until the process exits; a trace whose scratch
+ * does not fit is rejected with HX_ERR_INVALID and a message giving the
+ * bytes it would need.  Fewer warps run when the trace is large, so results
+ * are the same as hx_sim_run's but throughput is lower.
+ *
+ * The first call on a device looks up that device's address of the array
+ * (cudaGetSymbolAddress, with that device current); make it before any stream
+ * capture.  Runs on `stream` and returns when the results are in `results`.
+ * Every call on a device shares the one array: calls that overlap on the GPU
+ * (other threads, other streams) race and corrupt each other. */
+int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluster, const hx_grid* grid,
+                      int32_t objective, hx_result* results, hx_best* best, void* stream);
+
 typedef struct hx_info {
   int64_t n_sims;
   int64_t n_calls_total;

@@ -7,6 +7,7 @@
 #include <cstdio>
 #include <cstddef>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <string>
 #include <vector>
@@ -625,3 +626,245 @@ int hx_sim_destroy(hx_sim* h) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// hx_sim_run_static: the whole path for one trace without allocating memory.
+//
+// For callers that may not allocate device memory -- code running where
+// cudaMalloc is forbidden or unavailable (a host process that only owns
+// pre-arranged memory, a plugin whose host application controls every
+// allocation, a latency-critical loop that must not hit the allocator) -- this
+// entry point runs the same preparation, simulation and best-point kernels as
+// hx_sim_run, but every intermediate buffer (the copied inputs, the per-call
+// records, the per-warp heap arenas, the results) is carved from one
+// file-scope device array of HX_STATIC_SCRATCH_BYTES.  That array exists on
+// every GPU that loads this library, for as long as the library stays loaded.
+namespace {
+
+__device__ __align__(256) unsigned char hx_static_scratch[HX_STATIC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mu;
+unsigned char* g_static_base[kMaxDevices] = {};
+
+// Device address of hx_static_scratch on the current device, looked up once
+// per device (the host-side symbol is only a stand-in and must never be
+// passed to a kernel).
+int static_base(unsigned char** out) {
+  int dev = 0;
+  HX_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return fail(HX_ERR_INVALID, "device index out of range");
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_base[dev]) {
+    void* p = nullptr;
+    HX_CUDA(cudaGetSymbolAddress(&p, hx_static_scratch));
+    g_static_base[dev] = static_cast<unsigned char*>(p);
+  }
+  *out = g_static_base[dev];
+  return HX_OK;
+}
+
+__global__ void hx_widen_kernel(const int32_t* src, int64_t* dst, int64_t n) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) dst[i] = src[i];
+}
+
+// Bump carving of the static array; offsets are 256-byte aligned.
+struct Carve {
+  int64_t used = 0;
+  template <class T>
+  int64_t take(int64_t count) {
+    const int64_t off = used;
+    used = align_up(used + std::max<int64_t>(count, 1) * (int64_t)sizeof(T), 256);
+    return off;
+  }
+};
+
+}  // namespace
+
+extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluster, const hx_grid* grid,
+                                 int32_t objective, hx_result* results, hx_best* best, void* stream) {
+  g_err.clear();
+  if (!trace || !results) return fail(HX_ERR_INVALID, "trace and results must not be NULL");
+  if (objective != HX_OBJ_P95 && objective != HX_OBJ_P95_SLO95) return fail(HX_ERR_INVALID, "unknown objective");
+  int64_t min_prefill = 0, max_decode = 0;
+  int rc;
+  if ((rc = validate_cluster(cluster, &min_prefill, &max_decode))) return rc;
+  if ((rc = validate_grid(grid))) return rc;
+  if ((rc = validate_trace(trace, 0, cluster, min_prefill, max_decode))) return rc;
+  const int64_t nq = trace->n_queries, nc = trace->n_calls, P = grid->n_points;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  hx::ClusterK ck{};
+  ck.n_inst = cluster->n_inst;
+  ck.n_types = cluster->n_types;
+  ck.ref_type = cluster->ref_type;
+  ck.rmax = cluster->rmax;
+  ck.slo_mult_fp = cluster->slo_mult_fp;
+  for (int t = 0; t < HX_MAX_TYPES; ++t) {
+    const bool on = t < cluster->n_types;
+    ck.prefill[t] = on ? cluster->prefill_tok_s[t] : 1;
+    ck.decode[t] = on ? cluster->decode_us_tok[t] : 0;
+    ck.slots[t] = on ? cluster->slots[t] : 0;
+    ck.cnt[t] = 0;
+  }
+  for (int st = 0; st < 4; ++st) {
+    ck.ref_prompt[st] = cluster->stage_ref_prompt[st];
+    ck.ref_out[st] = cluster->stage_ref_out[st];
+  }
+  int base = 0;
+  for (int m = 0; m < HX_MAX_INST; ++m) {
+    const bool on = m < cluster->n_inst;
+    const int ty = on ? cluster->inst_type[m] : 0;
+    ck.inst_type[m] = (uint8_t)ty;
+    ck.inst_slots[m] = on ? (uint8_t)cluster->slots[ty] : 0;
+    ck.slot_base[m] = (uint16_t)base;
+    if (on) {
+      base += cluster->slots[ty];
+      ck.cnt[ty]++;
+    }
+  }
+  ck.total_slots = base;
+  ck.smem_per_warp = per_warp_smem(base);
+
+  // layout of the static array: inputs, records, results, then per-warp scratch
+  Carve cv;
+  const int64_t o_qoff = cv.take<int64_t>(2), o_coff = cv.take<int64_t>(2), o_ctr = cv.take<unsigned long long>(1);
+  const int64_t o_arr = cv.take<int64_t>(nq), o_k = cv.take<uint8_t>(nq), o_cb32 = cv.take<int32_t>(nq + 1);
+  const int64_t o_qcall = cv.take<int64_t>(nq + 1);
+  const int64_t o_prompt = cv.take<int32_t>(nc), o_out = cv.take<int32_t>(nc), o_oest = cv.take<int32_t>(nc);
+  const int64_t o_stage = cv.take<uint8_t>(nc), o_cand = cv.take<uint8_t>(nc), o_retry = cv.take<uint8_t>(nc);
+  const int64_t o_alpha = cv.take<int64_t>(P), o_gamma = cv.take<int64_t>(P), o_beta = cv.take<int64_t>(P);
+  const int64_t o_rho = cv.take<int32_t>(P), o_lp = cv.take<uint8_t>(P), o_dp = cv.take<uint8_t>(P);
+  const int64_t o_rec = cv.take<hx::CallRec>(nc), o_res = cv.take<hx_result>(P);
+  const int64_t o_bt = cv.take<hx::BestCand>(2), o_bg = cv.take<hx::BestCand>(2);
+  const int64_t fixed = cv.used;
+  const int32_t kcap = (int32_t)(nq - (95 * nq + 99) / 100 + 1);
+  const int64_t arena_per_warp = 4 * nc + 16 * HX_MAX_INST;
+  const int64_t chains_per_warp = align_up(std::max<int64_t>(nq, 1), 256);
+  const int64_t topk_per_warp = align_up(std::max<int32_t>(kcap, 1), 32);
+  const int64_t per_warp = align_up(arena_per_warp * (int64_t)sizeof(hx::HeapEnt), 256) + chains_per_warp +
+                           align_up(topk_per_warp * 8, 256);
+  const int64_t room = (int64_t)HX_STATIC_SCRATCH_BYTES - fixed;
+  const int64_t fit_warps = room > 0 ? room / per_warp : 0;
+  if (fit_warps < hx::kWarpsPerBlock)
+    return fail(HX_ERR_INVALID, "trace too large for the static scratch: it needs " +
+                                    std::to_string(fixed + hx::kWarpsPerBlock * per_warp) + " bytes, the array holds " +
+                                    std::to_string((int64_t)HX_STATIC_SCRATCH_BYTES));
+
+  int dev = 0;
+  cudaDeviceProp prop;
+  HX_CUDA(cudaGetDevice(&dev));
+  HX_CUDA(cudaGetDeviceProperties(&prop, dev));
+  const int smem_per_block = hx::kWarpsPerBlock * ck.smem_per_warp;
+  HX_CUDA(cudaFuncSetAttribute(hx::hx_sim_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_per_block));
+  int bps = 0;
+  HX_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, hx::hx_sim_kernel, hx::kWarpsPerBlock * 32,
+                                                        smem_per_block));
+  if (bps < 1) return fail(HX_ERR_CUDA, "simulation kernel does not fit on an SM");
+  int64_t blocks = std::min<int64_t>((int64_t)bps * prop.multiProcessorCount, fit_warps / hx::kWarpsPerBlock);
+  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (P + hx::kWarpsPerBlock - 1) / hx::kWarpsPerBlock));
+  const int64_t warps = blocks * hx::kWarpsPerBlock;
+  const int64_t o_arena = fixed;
+  const int64_t o_chains = o_arena + warps * align_up(arena_per_warp * (int64_t)sizeof(hx::HeapEnt), 256);
+  const int64_t o_topk = o_chains + warps * chains_per_warp;
+
+  unsigned char* sb = nullptr;
+  if ((rc = static_base(&sb))) return rc;
+  auto at = [&](int64_t off) { return static_cast<void*>(sb + off); };
+  const int64_t offs[4] = {0, nq, 0, nc};
+  HX_CUDA(cudaMemcpyAsync(at(o_qoff), offs, 2 * sizeof(int64_t), cudaMemcpyHostToDevice, s));
+  HX_CUDA(cudaMemcpyAsync(at(o_coff), offs + 2, 2 * sizeof(int64_t), cudaMemcpyHostToDevice, s));
+  struct Up {
+    int64_t off;
+    const void* src;
+    int64_t bytes;
+  } ups[] = {{o_arr, trace->arrival_us, nq * 8},     {o_k, trace->k, nq},
+             {o_cb32, trace->call_base, (nq + 1) * 4}, {o_prompt, trace->prompt, nc * 4},
+             {o_out, trace->out, nc * 4},             {o_oest, trace->out_est, nc * 4},
+             {o_stage, trace->stage, nc},             {o_cand, trace->cand, nc},
+             {o_retry, trace->retry, nc},             {o_alpha, grid->alpha_fp, P * 8},
+             {o_gamma, grid->gamma_fp, P * 8},        {o_beta, grid->beta_us2, P * 8},
+             {o_rho, grid->rho, P * 4},               {o_lp, grid->local_policy, P},
+             {o_dp, grid->dispatch_policy, P}};
+  for (const Up& u : ups)
+    if (u.bytes > 0) HX_CUDA(cudaMemcpyAsync(at(u.off), u.src, (size_t)u.bytes, cudaMemcpyHostToDevice, s));
+  hx_widen_kernel<<<(unsigned)std::max<int64_t>(1, (nq + 1 + 255) / 256), 256, 0, s>>>(
+      static_cast<const int32_t*>(at(o_cb32)), static_cast<int64_t*>(at(o_qcall)), nq + 1);
+  HX_CUDA(cudaGetLastError());
+
+  hx::PrepArgs pa;
+  pa.arrival = static_cast<const int64_t*>(at(o_arr));
+  pa.kq = static_cast<const uint8_t*>(at(o_k));
+  pa.qcall = static_cast<const int64_t*>(at(o_qcall));
+  pa.q_off = static_cast<const int64_t*>(at(o_qoff));
+  pa.c_off = static_cast<const int64_t*>(at(o_coff));
+  pa.prompt = static_cast<const int32_t*>(at(o_prompt));
+  pa.out = static_cast<const int32_t*>(at(o_out));
+  pa.out_est = static_cast<const int32_t*>(at(o_oest));
+  pa.stage = static_cast<const uint8_t*>(at(o_stage));
+  pa.cand = static_cast<const uint8_t*>(at(o_cand));
+  pa.retry = static_cast<const uint8_t*>(at(o_retry));
+  pa.n_queries = nq;
+  pa.n_traces = 1;
+  pa.rec = static_cast<hx::CallRec*>(at(o_rec));
+  pa.work_counter = static_cast<unsigned long long*>(at(o_ctr));  // zeroed by the prep kernel
+
+  hx::SimArgs sa;
+  sa.rec = pa.rec;
+  sa.arrival = pa.arrival;
+  sa.qcall = pa.qcall;
+  sa.q_off = pa.q_off;
+  sa.c_off = pa.c_off;
+  sa.alpha = static_cast<const int64_t*>(at(o_alpha));
+  sa.gamma = static_cast<const int64_t*>(at(o_gamma));
+  sa.rho = static_cast<const int32_t*>(at(o_rho));
+  sa.beta = static_cast<const int64_t*>(at(o_beta));
+  sa.lpol = static_cast<const uint8_t*>(at(o_lp));
+  sa.dpol = static_cast<const uint8_t*>(at(o_dp));
+  sa.n_points = (int32_t)P;
+  sa.n_traces = 1;
+  sa.n_sims = P;
+  sa.results = static_cast<hx_result*>(at(o_res));
+  sa.work_counter = pa.work_counter;
+  sa.arena = static_cast<hx::HeapEnt*>(at(o_arena));
+  sa.arena_per_warp = align_up(arena_per_warp * (int64_t)sizeof(hx::HeapEnt), 256) / (int64_t)sizeof(hx::HeapEnt);
+  sa.chains = static_cast<uint8_t*>(at(o_chains));
+  sa.chains_per_warp = chains_per_warp;
+  sa.topk = static_cast<int64_t*>(at(o_topk));
+  sa.topk_per_warp = align_up(topk_per_warp * 8, 256) / 8;
+  sa.rec_map = nullptr;
+  sa.rec_inst = nullptr;
+  sa.rec_enq = nullptr;
+  sa.rec_budget = nullptr;
+  sa.rec_start = nullptr;
+  sa.rec_stride = 0;
+
+  hx::BestArgs ba;
+  ba.results = sa.results;
+  ba.q_off = pa.q_off;
+  ba.n_traces = 1;
+  ba.n_points = (int32_t)P;
+  ba.per_trace = static_cast<hx::BestCand*>(at(o_bt));
+  ba.global = static_cast<hx::BestCand*>(at(o_bg));
+
+  hx::hx_prep_kernel<<<(unsigned)std::max<int64_t>(1, (nq + 255) / 256), 256, 0, s>>>(pa, ck);
+  HX_CUDA(cudaGetLastError());
+  hx::hx_sim_kernel<<<(unsigned)blocks, hx::kWarpsPerBlock * 32, smem_per_block, s>>>(sa, ck);
+  HX_CUDA(cudaGetLastError());
+  hx::hx_best_kernel<<<2, 256, 0, s>>>(ba);
+  HX_CUDA(cudaGetLastError());
+  HX_CUDA(cudaMemcpyAsync(results, at(o_res), (size_t)P * sizeof(hx_result), cudaMemcpyDeviceToHost, s));
+  hx::BestCand bg[2];
+  HX_CUDA(cudaMemcpyAsync(bg, at(o_bg), sizeof(bg), cudaMemcpyDeviceToHost, s));
+  HX_CUDA(cudaStreamSynchronize(s));
+  if (best) {
+    const bool v = bg[objective].flags & 1;
+    best->global_point = v ? bg[objective].p : -1;
+    best->pad = 0;
+    best->global_sum_p95 = v ? bg[objective].p95 : -1;
+    best->global_slo_met = v ? bg[objective].slo : -1;
+    if (best->per_trace_point) best->per_trace_point[0] = best->global_point;
+  }
+  return HX_OK;
+}

@@ -101,7 +101,8 @@ def load(path: Optional[str] = None):
                        ("hx_sim_run", [vp, vp]), ("hx_sim_results", [vp, vp, sz]),
                        ("hx_sim_best", [vp, i32, vp]), ("hx_sim_records", [vp, i32, vp, vp, vp, vp, sz]),
                        ("hx_sim_prep", [vp, i32, vp, vp, vp, vp, sz]), ("hx_sim_timings", [vp, vp, vp, vp]),
-                       ("hx_sim_info", [vp, vp]), ("hx_sim_destroy", [vp])]:
+                       ("hx_sim_info", [vp, vp]), ("hx_sim_destroy", [vp]),
+                       ("hx_sim_run_static", [vp, vp, vp, i32, vp, vp, vp])]:
         fn = getattr(lib, name)
         fn.restype = ctypes.c_int
         fn.argtypes = args
@@ -144,6 +145,35 @@ class _Traces:
                     _c(t.stage, np.uint8), _c(t.cand, np.uint8), _c(t.retry, np.uint8)]
             self.keep.append(cols)
             self.arr[i] = hx_trace(int(cols[0].shape[0]), int(cols[3].shape[0]), *[_p(x) for x in cols])
+
+
+def _cluster_struct(c):
+    cols = [_c(c.prefill_tok_s, np.int32), _c(c.decode_us_tok, np.int32), _c(c.slots, np.int32),
+            _c(c.inst_type, np.uint8), _c(c.stage_ref_prompt, np.int32), _c(c.stage_ref_out, np.int32)]
+    st = hx_cluster(int(cols[0].shape[0]), _p(cols[0]), _p(cols[1]), _p(cols[2]), int(cols[3].shape[0]),
+                    _p(cols[3]), int(c.ref_type), int(c.slo_mult_fp), int(c.rmax), _p(cols[4]), _p(cols[5]))
+    return st, cols
+
+
+def _grid_struct(g):
+    cols = [_c(g.alpha_fp, np.int64), _c(g.gamma_fp, np.int64), _c(g.rho, np.int32), _c(g.beta_us2, np.int64),
+            _c(g.local_policy, np.uint8), _c(g.dispatch_policy, np.uint8)]
+    return hx_grid(int(cols[0].shape[0]), *[_p(x) for x in cols]), cols
+
+
+def run_static(trace, cluster, grid, objective: int = OBJ_P95, stream=None):
+    """hx_sim_run_static: one trace through the whole path with no memory
+    allocation (the library's fixed device array holds every intermediate).
+    Returns (results, (best point, its P95, its SLO count))."""
+    lib = load()
+    tr = _Traces([trace])
+    hc, keep_c = _cluster_struct(cluster)
+    hg, keep_g = _grid_struct(grid)
+    res = np.zeros(int(grid.alpha_fp.shape[0]), RESULT_DTYPE)
+    best = hx_best(0, 0, 0, 0, None)
+    _check(lib, lib.hx_sim_run_static(ctypes.cast(tr.arr, ctypes.c_void_p), ctypes.byref(hc), ctypes.byref(hg),
+                                      int(objective), _p(res), ctypes.byref(best), _stream_handle(stream)))
+    return res, (int(best.global_point), int(best.global_sum_p95), int(best.global_slo_met))
 
 
 class Sim:
