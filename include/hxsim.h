@@ -221,6 +221,13 @@ int hx_sim_timings(hx_sim* h, float* prep_ms, float* sim_ms, float* best_ms);
 int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluster, const hx_grid* grid,
                       int32_t objective, hx_result* results, hx_best* best, void* stream);
 
+/* Self-test of the library's device integer division (the reward and budget
+ * quotients): divides count pairs (host arrays, n < 2^63, 1 <= d < 2^54) on
+ * the current device with the library's routine into q and with the
+ * compiler's 64-bit division into q_ref.  Allocates and frees its own device
+ * buffers; synchronous. */
+int hx_selftest_div(const uint64_t* n, const uint64_t* d, uint64_t* q, uint64_t* q_ref, size_t count);
+
 typedef struct hx_info {
   int64_t n_sims;
   int64_t n_calls_total;

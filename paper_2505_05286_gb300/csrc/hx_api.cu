@@ -603,6 +603,29 @@ int hx_sim_timings(hx_sim* h, float* prep_ms, float* sim_ms, float* best_ms) {
   return HX_OK;
 }
 
+int hx_selftest_div(const uint64_t* n, const uint64_t* d, uint64_t* q, uint64_t* q_ref, size_t count) {
+  if (!n || !d || !q || !q_ref) return fail(HX_ERR_INVALID, "NULL argument");
+  for (size_t i = 0; i < count; ++i)
+    if (n[i] >= (uint64_t(1) << 63) || d[i] < 1 || d[i] >= (uint64_t(1) << 54))
+      return fail(HX_ERR_INVALID, "operands must satisfy n < 2^63 and 1 <= d < 2^54");
+  if (count == 0) return HX_OK;
+  uint64_t* buf = nullptr;
+  HX_CUDA(cudaMalloc(&buf, 4 * count * sizeof(uint64_t)));
+  auto run = [&]() -> int {
+    HX_CUDA(cudaMemcpy(buf, n, count * 8, cudaMemcpyHostToDevice));
+    HX_CUDA(cudaMemcpy(buf + count, d, count * 8, cudaMemcpyHostToDevice));
+    hx::hx_selftest_div_kernel<<<(unsigned)((count + 255) / 256), 256>>>(buf, buf + count, buf + 2 * count,
+                                                                         buf + 3 * count, (int64_t)count);
+    HX_CUDA(cudaGetLastError());
+    HX_CUDA(cudaMemcpy(q, buf + 2 * count, count * 8, cudaMemcpyDeviceToHost));
+    HX_CUDA(cudaMemcpy(q_ref, buf + 3 * count, count * 8, cudaMemcpyDeviceToHost));
+    return HX_OK;
+  };
+  const int rc = run();
+  cudaFree(buf);
+  return rc;
+}
+
 int hx_sim_info(hx_sim* h, hx_info* out) {
   if (!h || !out) return fail(HX_ERR_INVALID, "NULL argument");
   out->n_sims = h->n_sims;

@@ -148,5 +148,7 @@ struct BestArgs {
 __global__ void hx_prep_kernel(PrepArgs a, ClusterK c);
 __global__ void hx_sim_kernel(SimArgs a, ClusterK c);
 __global__ void hx_best_kernel(BestArgs a);
+__global__ void hx_selftest_div_kernel(const uint64_t* n, const uint64_t* d, uint64_t* q, uint64_t* q_ref,
+                                       int64_t count);
 
 }  // namespace hx

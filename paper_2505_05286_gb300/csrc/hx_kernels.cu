@@ -50,6 +50,41 @@ __device__ __forceinline__ int warp_argmax_s64(int64_t s, int idx) {
   return (int)__reduce_min_sync(kFull, c2 ? (uint32_t)idx : 0xffffffffu);
 }
 
+// floor(n / d) for 0 <= n < 2^63 and 1 <= d < 2^54.  Trial-quotient method
+// (Knuth, TAOCP vol. 2, 4.3.1): a quotient estimate from a single-precision
+// reciprocal, refined once on the exact int64 remainder, then corrected by at
+// most one step each way.  Operands reach float through two 32-bit halves.
+// Estimate error: |q0 - n/d| < 2^30 * 2^-21 + 1, so the remainder fits int64
+// and the refined quotient is within one of n/d.  Quotients of 2^30 or more
+// (and d = 1) take the exact integer paths.
+__device__ __forceinline__ float u64_to_float(uint64_t x) {
+  return __fmaf_rn((float)(uint32_t)(x >> 32), 4294967296.0f, (float)(uint32_t)x);
+}
+
+__device__ __forceinline__ float s64_to_float(int64_t x) {
+  return x < 0 ? -u64_to_float((uint64_t)(-x)) : u64_to_float((uint64_t)x);
+}
+
+__device__ __forceinline__ uint64_t udiv_trial(uint64_t n, uint64_t d) {
+  if (d == 1) return n;
+  float rd;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(rd) : "f"(u64_to_float(d)));
+  const float qf = u64_to_float(n) * rd;
+  if (qf >= 1073741824.0f) return n / d;
+  uint64_t q = (uint32_t)qf;
+  int64_t r = (int64_t)(n - q * d);
+  q += (int64_t)(int32_t)(s64_to_float(r) * rd);
+  r = (int64_t)(n - q * d);
+  if (r < 0) {
+    q--;
+    r += (int64_t)d;
+  } else if (r >= (int64_t)d) {
+    q++;
+    r -= (int64_t)d;
+  }
+  return q;
+}
+
 // Workload-balanced reward term of Eq. (score): beta / max(t_queue, 1), capped.
 __device__ __forceinline__ int64_t reward_of(int64_t beta, int64_t q) {
   int64_t r = beta / (q > 1 ? q : 1);
@@ -556,7 +591,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
           if (dirty0) { n = beta; d = q0 > 1 ? q0 : 1; job = 1; }
           else if (dirty1) { n = beta; d = q1 > 1 ? q1 : 1; job = 2; }
           else if (lane == cand) { n = (uint64_t)(num < 0 ? -num : num) * (uint64_t)tb; d = (uint64_t)dd; job = 3; }
-          const uint64_t res = n / d;
+          const uint64_t res = udiv_trial(n, d);
           const int64_t capped = res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap;
           if (job == 1) { rew0 = capped; dirty0 = false; }
           else if (job == 2) { rew1 = capped; dirty1 = false; }
@@ -754,6 +789,16 @@ __global__ void __launch_bounds__(256) hx_best_kernel(BestArgs a) {
         if (cand_better(x, mine[o], o)) mine[o] = x;
     }
     block_reduce_best(mine, a.global);
+  }
+}
+
+// Self-test of udiv_trial against the compiler's division.
+__global__ void hx_selftest_div_kernel(const uint64_t* n, const uint64_t* d, uint64_t* q, uint64_t* q_ref,
+                                       int64_t count) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < count) {
+    q[i] = udiv_trial(n[i], d[i]);
+    q_ref[i] = n[i] / d[i];
   }
 }
 

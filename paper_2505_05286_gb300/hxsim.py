@@ -102,7 +102,8 @@ def load(path: Optional[str] = None):
                        ("hx_sim_best", [vp, i32, vp]), ("hx_sim_records", [vp, i32, vp, vp, vp, vp, sz]),
                        ("hx_sim_prep", [vp, i32, vp, vp, vp, vp, sz]), ("hx_sim_timings", [vp, vp, vp, vp]),
                        ("hx_sim_info", [vp, vp]), ("hx_sim_destroy", [vp]),
-                       ("hx_sim_run_static", [vp, vp, vp, i32, vp, vp, vp])]:
+                       ("hx_sim_run_static", [vp, vp, vp, i32, vp, vp, vp]),
+                       ("hx_selftest_div", [vp, vp, vp, vp, sz])]:
         fn = getattr(lib, name)
         fn.restype = ctypes.c_int
         fn.argtypes = args
@@ -145,6 +146,17 @@ class _Traces:
                     _c(t.stage, np.uint8), _c(t.cand, np.uint8), _c(t.retry, np.uint8)]
             self.keep.append(cols)
             self.arr[i] = hx_trace(int(cols[0].shape[0]), int(cols[3].shape[0]), *[_p(x) for x in cols])
+
+
+def selftest_div(n: np.ndarray, d: np.ndarray):
+    """(library quotients, compiler quotients) of n // d on the current device."""
+    lib = load()
+    n = _c(n, np.uint64)
+    d = _c(d, np.uint64)
+    q = np.zeros_like(n)
+    qr = np.zeros_like(n)
+    _check(lib, lib.hx_selftest_div(_p(n), _p(d), _p(q), _p(qr), int(n.shape[0])))
+    return q, qr
 
 
 def _cluster_struct(c):
