@@ -122,6 +122,12 @@ struct WarpShared {
   // per-simulation constants
   int64_t A, one_minus_a, G, beta, f_s, f_g, cref_c, cref_e;
   int32_t rho, rmax, lpol, dpol, recj, kcap, rr, bump;
+  // this warp's scratch slices and the current trace's offsets
+  HeapEnt* arena;
+  uint8_t* chains;
+  int64_t* topk;
+  int64_t qb, cb;
+  int32_t nq, pad0;
   // lane-0 accumulators
   uint64_t digest;
   int64_t makespan;

@@ -311,10 +311,6 @@ __device__ __noinline__ void topk_insert(int64_t* h, int& n, int kcap, int64_t v
   }
 }
 
-__device__ __forceinline__ void prefetch_l1(const void* p) {
-  asm volatile("prefetch.global.L1 [%0];" ::"l"(p));
-}
-
 // Queue this event's dispatches to instance m (pending entries on the lanes of
 // mask pm) in m's heap, re-homing the heap in the arena when it is full.
 // All lanes call.  Returns HX_OK or HX_ERR_CAPACITY.
@@ -382,10 +378,13 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   WarpShared* const W = reinterpret_cast<WarpShared*>(smem_raw + warp * c.smem_per_warp);
-  const int64_t gw = (int64_t)blockIdx.x * kWarpsPerBlock + warp;
-  HeapEnt* const arena = a.arena + gw * a.arena_per_warp;
-  uint8_t* const chains = a.chains + gw * a.chains_per_warp;
-  int64_t* const topk = a.topk + gw * a.topk_per_warp;
+  if (lane == 0) {
+    // this warp's slices of the scratch arrays (kept in shared memory to spare registers)
+    const int64_t gw = (int64_t)blockIdx.x * kWarpsPerBlock + warp;
+    W->arena = a.arena + gw * a.arena_per_warp;
+    W->chains = a.chains + gw * a.chains_per_warp;
+    W->topk = a.topk + gw * a.topk_per_warp;
+  }
   const int N = c.n_inst;
   const int m0 = lane, m1 = lane + 32;
   const bool valid0 = m0 < N, valid1 = m1 < N;
@@ -408,6 +407,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
     const int64_t cb = a.c_off[t];
     const int32_t nc = (int32_t)(a.c_off[t + 1] - cb);
     const CallRec* const rec = a.rec + cb;
+    if (lane == 0) {
+      W->qb = qb;
+      W->cb = cb;
+      W->nq = nq;
+    }
 
     for (int m = lane; m < 64; m += 32) {
       W->nkey[m] = kKeyInf;
@@ -468,8 +472,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
     int64_t now = 0;
     int32_t status = HX_OK, npend = 0;
     uint64_t touched = 0;
-    const int32_t max_steps = nc + nq + 8;
-    int32_t steps = 0;
+    int32_t steps_left = nc + nq + 8;
 
     auto set_key = [&](int m, uint64_t nk) {
       if (lane == (m & 31)) {
@@ -481,7 +484,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
     for (;;) {
       const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
       if (ck == kKeyInf && akey == kKeyInf) break;
-      if (++steps > max_steps) {
+      if (--steps_left < 0) {
         status = HX_ERR_STEP_LIMIT;
         break;
       }
@@ -496,7 +499,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         const int sb = c.slot_base[m];
         const int sl = W->nslot[m];
         const int32_t rid = (int32_t)(W->slot[sb + sl] & 0xffffffull);
-        if (lane < 8 && rid + lane < nc) prefetch_l1(rec + rid + lane);
+        // the finished call's record: issued now, used after the slot rescan
+        const CallRec* r = rec + rid;
+        const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
+        const int64_t est_m = r->est[c.inst_type[m]];
+        const int hs_m = W->hsize[m];
         __syncwarp();
         if (lane == 0) {
           W->slot[sb + sl] = kKeyInf;
@@ -513,23 +520,21 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
           W->nslot[m] = who ? __ffs(who) - 1 : -1;
         }
         set_key(m, mk);
-        const CallRec* r = rec + rid;
-        const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
-        const int64_t est_m = r->est[c.inst_type[m]];
         if (lane == (m & 31)) {
           if (m < 32) { q0 -= est_m; dirty0 = true; }
           else { q1 -= est_m; dirty1 = true; }
         }
-        touched |= 1ull << m;
+        // the freed slot needs a batch boundary only if requests wait for it
+        if (hs_m > 0) touched |= 1ull << m;
         const int stg = tail.w & 0xff;
         const int32_t qid = tail.z;
         if (stg == HX_STAGE_S) {
           const int k = (tail.w >> 16) & 0xff;
-          if (lane == 0) chains[qid] = (uint8_t)k;
+          if (lane == 0) W->chains[qid] = (uint8_t)k;
           rel_first = rid + 1;
           rel_count = k;
         } else if (stg == HX_STAGE_E) {
-          if (lane == 0) finish_query(W, topk, qid, now, r->arrival, r->deadline);
+          if (lane == 0) finish_query(W, W->topk, qid, now, r->arrival, r->deadline);
         } else {
           const int32_t nx = tail.y;
           if (nx >= 0) {
@@ -538,6 +543,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
           } else {
             int left = 0;
             if (lane == 0) {
+              uint8_t* const chains = W->chains;
               left = chains[qid] - 1;
               chains[qid] = (uint8_t)left;
             }
@@ -548,10 +554,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         }
       } else {
         now = (int64_t)(akey >> 7);
-        rel_first = (int32_t)(a.qcall[qb + qa] - cb);
+        const int64_t qbase = W->qb;
+        rel_first = (int32_t)(a.qcall[qbase + qa] - W->cb);
         rel_count = 1;
         qa++;
-        akey = qa < nq ? (((uint64_t)a.arrival[qb + qa] << 7) | kArrivalTag) : kKeyInf;
+        akey = qa < W->nq ? (((uint64_t)a.arrival[qbase + qa] << 7) | kArrivalTag) : kKeyInf;
       }
 
       // Sec. 4.1 + 4.2 for each released request, in request-id order: budget at
@@ -638,14 +645,16 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
       while (tm) {
         const int m = __ffsll((long long)tm) - 1;
         tm &= tm - 1;
-        const unsigned pm = __ballot_sync(kFull, lane < npend && pend_m == m);
         const uint32_t fm = W->freem[m];
         const int hs = W->hsize[m];
+        const uint64_t nkey0 = W->nkey[m];
+        const unsigned pm = __ballot_sync(kFull, lane < npend && pend_m == m);
         __syncwarp();
+        uint64_t nkey = nkey0;  // lane 0 tracks the instance's earliest (end, rid)
         // fast path: an empty queue with room for all of this event's arrivals
         const bool direct = hs == 0 && __popc(pm) <= __popc(fm);
         if (!direct && pm) {
-          status = push_pending(W, arena, a.arena_per_warp, m, pm, pend_key, pend_rid, pend_svc, lane);
+          status = push_pending(W, W->arena, a.arena_per_warp, m, pm, pend_key, pend_rid, pend_svc, lane);
           if (status != HX_OK) break;
         }
         unsigned bits = direct ? pm : 0u;
@@ -662,7 +671,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
             const bool go = W->freem[m] != 0u && n > 0;
             __syncwarp();
             if (!go) break;
-            const HeapEnt top = heap_pop_warp(arena + W->hoff[m], n, lane);
+            const HeapEnt top = heap_pop_warp(W->arena + W->hoff[m], n, lane);
             if (lane == 0) W->hsize[m] = n - 1;
             rid = top.rid;
             svc = top.svc;
@@ -675,7 +684,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
             W->freem[m] = fr & ~(1u << sl);
             const uint64_t nk = ((uint64_t)(now + svc) << 24) | (uint64_t)(uint32_t)rid;
             W->slot[sb + sl] = nk;
-            if (nk < W->nkey[m]) {
+            if (nk < nkey) {
+              nkey = nk;
               W->nkey[m] = nk;
               W->nslot[m] = sl;
             }
@@ -685,7 +695,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
           }
           __syncwarp();
         }
-        set_key(m, W->nkey[m]);
+        set_key(m, __shfl_sync(kFull, nkey, 0));
       }
       if (status != HX_OK) break;
     }
@@ -696,7 +706,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
       const int32_t n_done = W->n_done;
       if (st == HX_OK && n_done != nq) st = HX_ERR_STEP_LIMIT;
       hx_result res;
-      res.p95_us = st == HX_OK ? (nq > 0 ? topk[0] : 0) : -1;
+      res.p95_us = st == HX_OK ? (nq > 0 ? W->topk[0] : 0) : -1;
       res.makespan_us = W->makespan;
       res.events = W->events;
       res.digest = W->digest;
