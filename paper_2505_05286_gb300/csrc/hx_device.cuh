@@ -113,6 +113,7 @@ struct SimArgs {
 // slot state, per-simulation constants and lane-0 accumulators, then one
 // 64-bit (end << 24 | request id) key per batch slot of the cluster.
 struct WarpShared {
+  int64_t q[HX_MAX_INST];       // t_queue: Eq. comp summed over requests dispatched and unfinished
   uint64_t nkey[HX_MAX_INST];   // earliest running (end << 24 | rid), or all ones
   int32_t hoff[HX_MAX_INST];    // local queue: heap offset in the arena
   int32_t hcap[HX_MAX_INST];    //              heap capacity

@@ -370,7 +370,7 @@ __device__ __noinline__ int64_t budget_wide(int64_t num, int64_t tb, int64_t d) 
 }  // namespace
 
 #ifndef HX_SIM_MIN_BLOCKS
-#define HX_SIM_MIN_BLOCKS 6
+#define HX_SIM_MIN_BLOCKS 7
 #endif
 // Resident blocks per SM the register allocation aims for (4 warps each).
 __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim_kernel(SimArgs a, ClusterK c) {
@@ -459,7 +459,9 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
     __syncwarp();
 
     // this lane's instances: queue cost, cached reward and its staleness, event keys
-    int64_t q0 = 0, q1 = 0;
+    // (t_queue of instance m lives in W->q[m], touched only by its owner lane)
+    W->q[m0] = 0;
+    W->q[m1] = 0;
     int64_t rew0 = reward_of(W->beta, 0), rew1 = rew0;
     bool dirty0 = false, dirty1 = false;
     uint64_t k0 = kKeyInf, k1 = kKeyInf;
@@ -521,8 +523,9 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         }
         set_key(m, mk);
         if (lane == (m & 31)) {
-          if (m < 32) { q0 -= est_m; dirty0 = true; }
-          else { q1 -= est_m; dirty1 = true; }
+          W->q[m] -= est_m;
+          if (m < 32) dirty0 = true;
+          else dirty1 = true;
         }
         // the freed slot needs a batch boundary only if requests wait for it
         if (hs_m > 0) touched |= 1ull << m;
@@ -595,8 +598,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
           const int cand = (need_budget && ~busy) ? __ffs(~busy) - 1 : -1;
           uint64_t n = 0, d = 1;
           int job = 0;
-          if (dirty0) { n = beta; d = q0 > 1 ? q0 : 1; job = 1; }
-          else if (dirty1) { n = beta; d = q1 > 1 ? q1 : 1; job = 2; }
+          if (dirty0) { const int64_t q = W->q[m0]; n = beta; d = q > 1 ? q : 1; job = 1; }
+          else if (dirty1) { const int64_t q = W->q[m1]; n = beta; d = q > 1 ? q : 1; job = 2; }
           else if (lane == cand) { n = (uint64_t)(num < 0 ? -num : num) * (uint64_t)tb; d = (uint64_t)dd; job = 3; }
           const uint64_t res = udiv_trial(n, d);
           const int64_t capped = res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap;
@@ -623,8 +626,9 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         const int64_t est_m = pick4(e4, tym);
         const int svc_m = pick4(s4, tym);
         if (lane == (m & 31)) {
-          if (m < 32) { q0 += est_m; dirty0 = true; }
-          else { q1 += est_m; dirty1 = true; }
+          W->q[m] += est_m;
+          if (m < 32) dirty0 = true;
+          else dirty1 = true;
         }
         const long long key = W->lpol == HX_LOCAL_PQ ? (long long)(kScale * (est_m - budget) - W->G * now) : (long long)(-now);
         if (lane == npend) {
