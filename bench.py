@@ -30,6 +30,7 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+from paper_2505_05286_gb300 import dist as D  # noqa: E402
 from paper_2505_05286_gb300 import workloads as W  # noqa: E402
 
 CFG = 4
@@ -120,27 +121,10 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def _dist():
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return world, rank, local
-
-
 def _barrier(world):
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
-
-
-def _max_over_ranks(world, x: float) -> float:
-    if world == 1:
-        return x
-    import torch
-    import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
 
 
 def oracle_sample(wl, n_sims: int, seed: int, procs: int):
@@ -173,7 +157,7 @@ def cpu_baseline(wl, budget_s: float = 20.0):
 
 
 def run_reference(args):
-    world, rank, _ = _dist()
+    world, rank, _ = D.env()
     if rank != 0:
         return
     wl = W.make_workload(CFG)
@@ -203,7 +187,7 @@ def run_reference(args):
 
 def run_gpu(args):
     import torch
-    world, rank, local = _dist()
+    world, rank, local = D.env()
     if world > 1:
         import torch.distributed as dist
         torch.cuda.set_device(local)
@@ -214,7 +198,7 @@ def run_gpu(args):
     from paper_2505_05286_gb300 import hxsim as H
     B.build()
     # weak scaling: every rank simulates its own 256 traces (trace seeds offset by rank)
-    wl = W.make_workload(CFG, first_trace=rank * W.CONFIGS[CFG].n_traces)
+    wl = W.make_workload(CFG, first_trace=D.first_trace(rank, W.CONFIGS[CFG].n_traces))
     n_calls = wl.n_calls
     P = wl.grid.n_points
     sim = H.Sim(wl.traces, wl.cluster, wl.grid, timing=True)
@@ -239,7 +223,7 @@ def run_gpu(args):
     t_ms = start.elapsed_time(stop)
     # per-kernel times of the last timed step (events the library records on the same stream)
     sim_ms.append(sim.timings())
-    t_ms = _max_over_ranks(world, t_ms)
+    t_ms = D.max_over_ranks(t_ms)
     res = sim.results()
     ok = bool((res["status"] == 0).all())
     events_per_step = int(res["events"].sum())
@@ -263,10 +247,13 @@ def run_gpu(args):
         sim.run(stream)
         res2 = sim.results()
     torch.cuda.synchronize()
-    e2e_s = _max_over_ranks(world, time.perf_counter() - t0)
+    e2e_s = D.max_over_ranks(time.perf_counter() - t0)
     ok = ok and bool((res2["digest"] == res["digest"]).all())
     e2e_value = sims_total * e2e_steps / e2e_s
-    best = sim.best(wl.objective)
+    # best point of the whole job: per-point sums over every rank's traces
+    sp, ss, sf = sim.point_sums()
+    sp, ss, sf, nq_all = D.global_point_sums(sp, ss, sf, sum(t.n_queries for t in wl.traces))
+    best = H.best_of_sums(sp, ss, sf, nq_all, wl.objective)
 
     peaks, peak_kind = _peaks()
     clocks = clk.summary()

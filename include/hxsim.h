@@ -29,7 +29,8 @@
  *    of G, min(rho, R - u) corrections and E as applicable;
  *  - Eq. (priority) with ageing weight gamma: U = t_comp - t_slo + gamma*tau;
  *    at each batch boundary an instance starts its highest-U waiting request
- *    (ties to the lowest request id);
+ *    (ties to the lowest request id); alternatively FCFS, or LLF (the
+ *    query's laxity: deadline - now - the same remaining-path cost);
  *  - events in the order (time, completions before arrivals, instance,
  *    request id / query id);
  *  - per simulation the nearest-rank P95 of query latencies
@@ -64,7 +65,7 @@ enum {
 };
 
 enum { HX_STAGE_S = 0, HX_STAGE_G = 1, HX_STAGE_C = 2, HX_STAGE_E = 3 };
-enum { HX_LOCAL_PQ = 0, HX_LOCAL_FCFS = 1 };
+enum { HX_LOCAL_PQ = 0, HX_LOCAL_FCFS = 1, HX_LOCAL_LLF = 2 };
 enum { HX_DISPATCH_WB = 0, HX_DISPATCH_RR = 1 };
 enum { HX_OBJ_P95 = 0, HX_OBJ_P95_SLO95 = 1 };
 
@@ -115,7 +116,8 @@ typedef struct hx_grid {
   const int64_t* gamma_fp;          /* [n] 0..4*SCALE (urgency ageing weight) */
   const int32_t* rho;               /* [n] 0..15 corrections assumed by the budget */
   const int64_t* beta_us2;          /* [n] >= 0, beta = C_ref * Q_ref */
-  const uint8_t* local_policy;      /* [n] HX_LOCAL_* */
+  const uint8_t* local_policy;      /* [n] HX_LOCAL_*: urgency queue (Sec. 4.2), FCFS, or the
+                                       least-laxity-first baseline of Sec. 5.1 */
   const uint8_t* dispatch_policy;   /* [n] HX_DISPATCH_* */
 } hx_grid;
 
@@ -173,6 +175,19 @@ int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n);
 
 /* Wait for the last run and return the best point for `objective`. */
 int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out);
+
+/* Per-point sums over the handle's traces from the last run (the partial
+ * sums a rank contributes when traces are spread over several GPUs): summed
+ * P95, summed SLO hits, and the number of failed simulations, each
+ * [n_points] host arrays.  Waits for the run. */
+int hx_sim_point_sums(hx_sim* h, int64_t* sum_p95, int64_t* sum_slo_met, int32_t* n_failed, size_t n_points);
+
+/* The grid's best point (Sec. 4.3) from per-point sums added up over every
+ * rank's traces, with the same rules as hx_sim_best; n_queries_total is the
+ * number of queries behind the sums.  Runs the best-point kernel on the
+ * current device (allocating a small temporary buffer); synchronous. */
+int hx_best_of_sums(const int64_t* sum_p95, const int64_t* sum_slo_met, const int32_t* n_failed, int32_t n_points,
+                    int64_t n_queries_total, int32_t objective, hx_best* out);
 
 /* Per-call log of recorded simulation `rec_index` (position in
  * opt.record_sims): instance, dispatch time, SLO budget and start time of

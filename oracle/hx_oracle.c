@@ -24,6 +24,9 @@
  *    mean cost plus the stage reference costs of the rest of its own path
  *    (S -> G -> up to min(rho, R - u) corrections -> E);
  *  - urgency ages with weight gamma: U = t_comp - t_slo + gamma * tau;
+ *  - the LLF baseline of Sec. 5.1 orders waiting requests by the query's
+ *    laxity, deadline - now - remaining work, where the remaining work is
+ *    the same remaining-path cost as the budget denominator;
  *  - events are taken one at a time ordered by (time, completions before
  *    arrivals, instance, request id / query id); after each event the
  *    released successors are dispatched in request-id order, then every
@@ -75,22 +78,19 @@ static int64_t stage_ref(const hxo_cluster* cl, int s) {
   return sum / cl->n_inst;
 }
 
-/* splitmix64 finalizer (Steele, Lea & Flood 2014). */
-static uint64_t mix64(uint64_t z) {
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
-  return z ^ (z >> 31);
+/* Digest term of a (time, id << 8 | tag) pair:
+ * y = ((time * 0x9E3779B97F4A7C15) xor idtag) * 0xBF58476D1CE4E5B9, term = y xor (y >> 32). */
+static uint64_t digest_term(uint64_t t, uint64_t idtag) {
+  uint64_t y = ((t * 0x9E3779B97F4A7C15ULL) ^ idtag) * 0xBF58476D1CE4E5B9ULL;
+  return y ^ (y >> 32);
 }
 
-/* Digest terms: one finalizer over (time * golden ratio) xor (id << 8 | tag). */
-#define DIGEST_MUL 0x9E3779B97F4A7C15ULL
-
 static uint64_t call_term(int32_t rid, int inst, int64_t start) {
-  return mix64(((uint64_t)start * DIGEST_MUL) ^ (((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst));
+  return digest_term((uint64_t)start, ((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst);
 }
 
 static uint64_t query_term(int32_t qid, int64_t end) {
-  return mix64(((uint64_t)end * DIGEST_MUL) ^ (((uint64_t)(uint32_t)qid << 8) | 0xFFu));
+  return digest_term((uint64_t)end, ((uint64_t)(uint32_t)qid << 8) | 0xFFu);
 }
 
 static int cmp_i64(const void* a, const void* b) {
@@ -231,6 +231,7 @@ typedef struct {
   int32_t* inst;        /* per call */
   int64_t* enq;         /* per call */
   int64_t* budget;      /* per call */
+  int64_t* remaining;   /* per call: remaining-path cost at dispatch */
   int64_t* start;       /* per call */
   int64_t* end;         /* per call */
   int32_t* chains_left; /* per query */
@@ -272,7 +273,8 @@ static void dispatch(sim_t* s, int32_t c, int64_t now) {
   int32_t i = s->qid[c];
   int64_t tb = mean_est(tr, cl, c);
   int64_t elapsed = now - tr->arrival_us[i];
-  s->budget[c] = hxo_budget(s->t_slo[i], elapsed, tb, remaining_cost(s, c, tb));
+  s->remaining[c] = remaining_cost(s, c, tb);
+  s->budget[c] = hxo_budget(s->t_slo[i], elapsed, tb, s->remaining[c]);
   int best = -1;
   if (s->pt->dispatch_policy == 1) {
     best = (int)(s->rr_next % cl->n_inst);
@@ -312,15 +314,22 @@ static void fill_slots(sim_t* s, int64_t now, int64_t** ubuf, int64_t** ebuf, in
       }
       for (int32_t j = 0; j < w->n; ++j) {
         int32_t c = w->v[j];
-        /* Eq. (priority) with ageing weight gamma, in fixed point */
-        i128 u = (i128)FP_ONE * (est_on(tr, cl, m, c) - s->budget[c]) +
-                 (i128)s->pt->gamma_fp * (now - s->enq[c]);
+        i128 u;
+        if (s->pt->local_policy == 2) {
+          /* LLF (Sec. 5.1): least laxity first, as an urgency to maximise */
+          int32_t i = s->qid[c];
+          int64_t laxity = tr->arrival_us[i] + s->t_slo[i] - now - s->remaining[c];
+          u = -(i128)laxity;
+        } else {
+          /* Eq. (priority) with ageing weight gamma, in fixed point */
+          u = (i128)FP_ONE * (est_on(tr, cl, m, c) - s->budget[c]) + (i128)s->pt->gamma_fp * (now - s->enq[c]);
+        }
         if (u > (i128)INT64_MAX || u < (i128)INT64_MIN) s->bad = HXO_ERR_INVALID;
         (*ubuf)[j] = (int64_t)u;
         (*ebuf)[j] = s->enq[c];
         (*rbuf)[j] = c;
       }
-      int32_t j = hxo_pick(s->pt->local_policy, w->n, *rbuf, *ubuf, *ebuf);
+      int32_t j = hxo_pick(s->pt->local_policy == 1 ? 1 : 0, w->n, *rbuf, *ubuf, *ebuf);
       int32_t c = w->v[j];
       ivec_remove_at(w, j);
       if (!ivec_push(&s->running[m], c)) { s->bad = HXO_ERR_OOM; return; }
@@ -351,7 +360,7 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
   memset(res, 0, sizeof(*res));
   res->p95_us = -1;
   if (!validate(tr, cl) || pt->alpha_fp < 0 || pt->alpha_fp > FP_ONE || pt->beta_us2 < 0 ||
-      pt->gamma_fp < 0 || pt->rho < 0 || pt->local_policy < 0 || pt->local_policy > 1 ||
+      pt->gamma_fp < 0 || pt->rho < 0 || pt->local_policy < 0 || pt->local_policy > 2 ||
       pt->dispatch_policy < 0 || pt->dispatch_policy > 1) {
     res->status = HXO_ERR_INVALID;
     return HXO_ERR_INVALID;
@@ -370,6 +379,7 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
   s.inst = (int32_t*)calloc(nc1, sizeof(int32_t));
   s.enq = (int64_t*)calloc(nc1, sizeof(int64_t));
   s.budget = (int64_t*)calloc(nc1, sizeof(int64_t));
+  s.remaining = (int64_t*)calloc(nc1, sizeof(int64_t));
   s.start = (int64_t*)calloc(nc1, sizeof(int64_t));
   s.end = (int64_t*)calloc(nc1, sizeof(int64_t));
   s.q = (int64_t*)calloc((size_t)N, sizeof(int64_t));
@@ -383,7 +393,7 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
   int32_t* rbuf = NULL;
   int32_t bufcap = 0;
   int status = HXO_OK;
-  if (!s.t_slo || !s.chains_left || !s.qid || !s.state || !s.inst || !s.enq || !s.budget || !s.start ||
+  if (!s.t_slo || !s.chains_left || !s.qid || !s.state || !s.inst || !s.enq || !s.budget || !s.remaining || !s.start ||
       !s.end || !s.q || !s.waiting || !s.running || !lat || !est_tmp || !svc_tmp || !tbar_tmp) {
     status = HXO_ERR_OOM;
     goto done;
@@ -490,7 +500,7 @@ done:
   if (s.running)
     for (int m = 0; m < N; ++m) free(s.running[m].v);
   free(s.t_slo); free(s.chains_left); free(s.qid); free(s.state); free(s.inst); free(s.enq);
-  free(s.budget); free(s.start); free(s.end); free(s.q); free(s.waiting); free(s.running);
+  free(s.budget); free(s.remaining); free(s.start); free(s.end); free(s.q); free(s.waiting); free(s.running);
   free(lat); free(est_tmp); free(svc_tmp); free(tbar_tmp); free(ubuf); free(ebuf); free(rbuf);
   return status;
 }

@@ -50,7 +50,7 @@ typedef struct {
   int64_t gamma_fp;
   int64_t beta_us2;
   int32_t rho;
-  int32_t local_policy;     /* 0 = urgency PQ, 1 = FCFS */
+  int32_t local_policy;     /* 0 = urgency PQ, 1 = FCFS, 2 = least laxity first */
   int32_t dispatch_policy;  /* 0 = workload balanced, 1 = round robin */
 } hxo_point;
 

@@ -69,6 +69,7 @@ struct hx_sim {
   unsigned long long* d_counter = nullptr;
   hx::BestCand* d_best_trace = nullptr;
   hx::BestCand* d_best_global = nullptr;
+  int64_t* d_point_sums = nullptr;
   // device: scratch
   hx::HeapEnt* d_arena = nullptr;
   uint8_t* d_chains = nullptr;
@@ -156,7 +157,7 @@ int validate_grid(const hx_grid* g) {
     if (g->gamma_fp[p] < 0 || g->gamma_fp[p] > 4 * HX_SCALE) return fail(HX_ERR_INVALID, "gamma_fp must be 0..4*SCALE");
     if (g->rho[p] < 0 || g->rho[p] > HX_MAX_RETRY) return fail(HX_ERR_INVALID, "rho must be 0..15");
     if (g->beta_us2[p] < 0 || g->beta_us2[p] > (int64_t(1) << 62)) return fail(HX_ERR_INVALID, "beta_us2 out of range");
-    if (g->local_policy[p] > 1 || g->dispatch_policy[p] > 1) return fail(HX_ERR_INVALID, "unknown policy");
+    if (g->local_policy[p] > 2 || g->dispatch_policy[p] > 1) return fail(HX_ERR_INVALID, "unknown policy");
   }
   return HX_OK;
 }
@@ -349,7 +350,8 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
       (rc = h->alloc(&h->d_rho, h->n_points)) || (rc = h->alloc(&h->d_lp, h->n_points)) ||
       (rc = h->alloc(&h->d_dp, h->n_points)) || (rc = h->alloc(&h->d_rec, h->n_c)) ||
       (rc = h->alloc(&h->d_results, h->n_sims)) || (rc = h->alloc(&h->d_counter, 1)) ||
-      (rc = h->alloc(&h->d_best_trace, 2 * (int64_t)n_traces)) || (rc = h->alloc(&h->d_best_global, 2)))
+      (rc = h->alloc(&h->d_best_trace, 2 * (int64_t)n_traces)) || (rc = h->alloc(&h->d_best_global, 2)) ||
+      (rc = h->alloc(&h->d_point_sums, 3 * (int64_t)h->n_points)))
     return bail(rc);
   cudaStream_t s0 = nullptr;
   if ((rc = upload_traces(h, traces, s0)) || (rc = upload(h->d_q_off, q_off.data(), n_traces + 1, s0)) ||
@@ -499,6 +501,7 @@ int hx_sim_run(hx_sim* h, void* stream) {
   ba.n_points = h->n_points;
   ba.per_trace = h->d_best_trace;
   ba.global = h->d_best_global;
+  ba.point_sums = h->d_point_sums;
 
   const int prep_blocks = (int)std::max<int64_t>(1, (h->n_q + 255) / 256);
   if (h->timing) HX_CUDA(cudaEventRecord(h->ev[0], s));
@@ -546,6 +549,71 @@ int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out) {
     }
   }
   return HX_OK;
+}
+
+int hx_sim_point_sums(hx_sim* h, int64_t* sum_p95, int64_t* sum_slo_met, int32_t* n_failed, size_t n_points) {
+  if (!h || !sum_p95 || !sum_slo_met || !n_failed) return fail(HX_ERR_INVALID, "NULL argument");
+  if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
+  if ((int64_t)n_points != h->n_points) return fail(HX_ERR_INVALID, "n_points differs from the handle's");
+  HX_CUDA(cudaStreamSynchronize(h->last_stream));
+  std::vector<int64_t> v(3 * n_points);
+  HX_CUDA(cudaMemcpy(v.data(), h->d_point_sums, v.size() * sizeof(int64_t), cudaMemcpyDeviceToHost));
+  for (size_t p = 0; p < n_points; ++p) {
+    sum_p95[p] = v[3 * p];
+    sum_slo_met[p] = v[3 * p + 1];
+    n_failed[p] = (int32_t)v[3 * p + 2];
+  }
+  return HX_OK;
+}
+
+int hx_best_of_sums(const int64_t* sum_p95, const int64_t* sum_slo_met, const int32_t* n_failed, int32_t n_points,
+                    int64_t n_queries_total, int32_t objective, hx_best* out) {
+  if (!sum_p95 || !sum_slo_met || !n_failed || !out) return fail(HX_ERR_INVALID, "NULL argument");
+  if (n_points < 1 || n_queries_total < 0) return fail(HX_ERR_INVALID, "bad sizes");
+  if (objective != HX_OBJ_P95 && objective != HX_OBJ_P95_SLO95) return fail(HX_ERR_INVALID, "unknown objective");
+  // the summed table as one pseudo-trace, reduced by the same best-point kernel
+  std::vector<hx_result> table((size_t)n_points);
+  for (int32_t p = 0; p < n_points; ++p) {
+    if (sum_slo_met[p] < 0 || sum_slo_met[p] > INT32_MAX) return fail(HX_ERR_INVALID, "SLO sums out of range");
+    hx_result r{};
+    r.p95_us = sum_p95[p];
+    r.slo_met = (int32_t)sum_slo_met[p];
+    r.status = n_failed[p] ? HX_ERR_CAPACITY : HX_OK;
+    table[p] = r;
+  }
+  const int64_t qoff[2] = {0, n_queries_total};
+  void* buf = nullptr;
+  const size_t bytes = table.size() * sizeof(hx_result) + 2 * sizeof(int64_t) + 4 * sizeof(hx::BestCand);
+  HX_CUDA(cudaMalloc(&buf, bytes));
+  auto run = [&]() -> int {
+    unsigned char* b = static_cast<unsigned char*>(buf);
+    hx_result* d_res = reinterpret_cast<hx_result*>(b);
+    int64_t* d_qoff = reinterpret_cast<int64_t*>(b + table.size() * sizeof(hx_result));
+    hx::BestCand* d_cand = reinterpret_cast<hx::BestCand*>(d_qoff + 2);
+    HX_CUDA(cudaMemcpy(d_res, table.data(), table.size() * sizeof(hx_result), cudaMemcpyHostToDevice));
+    HX_CUDA(cudaMemcpy(d_qoff, qoff, sizeof(qoff), cudaMemcpyHostToDevice));
+    hx::BestArgs ba;
+    ba.results = d_res;
+    ba.q_off = d_qoff;
+    ba.n_traces = 1;
+    ba.n_points = n_points;
+    ba.per_trace = d_cand;
+    ba.global = d_cand + 2;
+    ba.point_sums = nullptr;
+    hx::hx_best_kernel<<<2, 256>>>(ba);
+    HX_CUDA(cudaGetLastError());
+    hx::BestCand g[2];
+    HX_CUDA(cudaMemcpy(g, d_cand + 2, sizeof(g), cudaMemcpyDeviceToHost));
+    const bool v = g[objective].flags & 1;
+    out->global_point = v ? g[objective].p : -1;
+    out->pad = 0;
+    out->global_sum_p95 = v ? g[objective].p95 : -1;
+    out->global_slo_met = v ? g[objective].slo : -1;
+    return HX_OK;
+  };
+  const int rc = run();
+  cudaFree(buf);
+  return rc;
 }
 
 int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us, int64_t* budget_us,
@@ -870,6 +938,7 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   ba.n_points = (int32_t)P;
   ba.per_trace = static_cast<hx::BestCand*>(at(o_bt));
   ba.global = static_cast<hx::BestCand*>(at(o_bg));
+  ba.point_sums = nullptr;
 
   hx::hx_prep_kernel<<<(unsigned)std::max<int64_t>(1, (nq + 255) / 256), 256, 0, s>>>(pa, ck);
   HX_CUDA(cudaGetLastError());

@@ -150,6 +150,7 @@ struct BestArgs {
   int32_t n_points;
   BestCand* per_trace;      // [T * 2]
   BestCand* global;         // [2]
+  int64_t* point_sums;      // [P * 3] (sum P95, sum SLO hits, failed sims) or NULL
 };
 
 __global__ void hx_prep_kernel(PrepArgs a, ClusterK c);

@@ -14,22 +14,23 @@ namespace hx {
 // ------------------------------------------------------------------ helpers
 __device__ __forceinline__ int64_t ceil_div_pos(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-// splitmix64 finalizer (Steele, Lea & Flood 2014), used for the digest.
-__device__ __forceinline__ uint64_t mix64(uint64_t z) {
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
+constexpr uint64_t kDigestMul = 0x9E3779B97F4A7C15ull;
+constexpr uint64_t kDigestMix = 0xBF58476D1CE4E5B9ull;
+
+// Digest terms: y = ((time * phi) xor (id << 8 | tag)) * c, term = y xor (y >> 32);
+// each step is a bijection, so a change of any one call's instance or start
+// (or any query's end) changes the sum.
+__device__ __forceinline__ uint64_t digest_term(uint64_t t, uint64_t idtag) {
+  const uint64_t y = ((t * kDigestMul) ^ idtag) * kDigestMix;
+  return y ^ (y >> 32);
 }
 
-constexpr uint64_t kDigestMul = 0x9E3779B97F4A7C15ull;
-
-// Digest terms: one finalizer over (time * golden ratio) xor (id << 8 | tag).
 __device__ __forceinline__ uint64_t call_term(int32_t rid, int inst, int64_t start) {
-  return mix64(((uint64_t)start * kDigestMul) ^ (((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst));
+  return digest_term((uint64_t)start, ((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst);
 }
 
 __device__ __forceinline__ uint64_t query_term(int32_t qid, int64_t end) {
-  return mix64(((uint64_t)end * kDigestMul) ^ (((uint64_t)(uint32_t)qid << 8) | 0xFFull));
+  return digest_term((uint64_t)end, ((uint64_t)(uint32_t)qid << 8) | 0xFFull);
 }
 
 __device__ __forceinline__ uint64_t warp_min_u64(uint64_t v) {
@@ -593,6 +594,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         bool need_budget = small;
         int bl = 0;
         const uint64_t beta = (uint64_t)W->beta;
+        if (W->one_minus_a == 0 || W->dpol == HX_DISPATCH_RR) {
+          // rewards carry no weight at alpha = 1 and are unused by round robin
+          dirty0 = false;
+          dirty1 = false;
+        }
         for (;;) {
           const unsigned busy = __ballot_sync(kFull, dirty0 || dirty1);
           const int cand = (need_budget && ~busy) ? __ffs(~busy) - 1 : -1;
@@ -630,7 +636,13 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
           if (m < 32) dirty0 = true;
           else dirty1 = true;
         }
-        const long long key = W->lpol == HX_LOCAL_PQ ? (long long)(kScale * (est_m - budget) - W->G * now) : (long long)(-now);
+        // local-queue key, higher first: Eq. (priority) aged by gamma with the
+        // common now dropped; FCFS: earliest enqueue; LLF: least deadline - now -
+        // remaining work, again with the common now dropped
+        const int lpol = W->lpol;
+        const long long key = lpol == HX_LOCAL_PQ     ? (long long)(kScale * (est_m - budget) - W->G * now)
+                              : lpol == HX_LOCAL_FCFS ? (long long)(-now)
+                                                      : (long long)(dd - dl);
         if (lane == npend) {
           pend_m = m;
           pend_key = key;
@@ -799,6 +811,11 @@ __global__ void __launch_bounds__(256) hx_best_kernel(BestArgs a) {
         valid &= r.status == HX_OK ? 1 : 0;
       }
       x.flags = valid | (x.slo * 100 >= 95 * nsum ? 2 : 0);
+      if (a.point_sums) {
+        a.point_sums[3 * p] = x.p95;
+        a.point_sums[3 * p + 1] = x.slo;
+        a.point_sums[3 * p + 2] = valid ? 0 : 1;
+      }
       for (int o = 0; o < 2; ++o)
         if (cand_better(x, mine[o], o)) mine[o] = x;
     }

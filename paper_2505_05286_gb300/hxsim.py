@@ -103,7 +103,9 @@ def load(path: Optional[str] = None):
                        ("hx_sim_prep", [vp, i32, vp, vp, vp, vp, sz]), ("hx_sim_timings", [vp, vp, vp, vp]),
                        ("hx_sim_info", [vp, vp]), ("hx_sim_destroy", [vp]),
                        ("hx_sim_run_static", [vp, vp, vp, i32, vp, vp, vp]),
-                       ("hx_selftest_div", [vp, vp, vp, vp, sz])]:
+                       ("hx_selftest_div", [vp, vp, vp, vp, sz]),
+                       ("hx_sim_point_sums", [vp, vp, vp, vp, sz]),
+                       ("hx_best_of_sums", [vp, vp, vp, i32, ctypes.c_int64, i32, vp])]:
         fn = getattr(lib, name)
         fn.restype = ctypes.c_int
         fn.argtypes = args
@@ -157,6 +159,16 @@ def selftest_div(n: np.ndarray, d: np.ndarray):
     qr = np.zeros_like(n)
     _check(lib, lib.hx_selftest_div(_p(n), _p(d), _p(q), _p(qr), int(n.shape[0])))
     return q, qr
+
+
+def best_of_sums(sum_p95, sum_slo_met, n_failed, n_queries_total: int, objective: int = OBJ_P95):
+    """Best point from per-point sums gathered over several handles or ranks."""
+    lib = load()
+    a, b, c = _c(sum_p95, np.int64), _c(sum_slo_met, np.int64), _c(n_failed, np.int32)
+    best = hx_best(0, 0, 0, 0, None)
+    _check(lib, lib.hx_best_of_sums(_p(a), _p(b), _p(c), int(a.shape[0]), int(n_queries_total), int(objective),
+                                    ctypes.byref(best)))
+    return int(best.global_point), int(best.global_sum_p95), int(best.global_slo_met)
 
 
 def _cluster_struct(c):
@@ -237,6 +249,14 @@ class Sim:
         b = hx_best(0, 0, 0, 0, _p(per))
         _check(self.lib, self.lib.hx_sim_best(self.h, int(objective), ctypes.byref(b)))
         return int(b.global_point), int(b.global_sum_p95), int(b.global_slo_met), per
+
+    def point_sums(self):
+        """(summed P95, summed SLO hits, failed simulations) per point over this handle's traces."""
+        a = np.zeros(self.n_points, np.int64)
+        b = np.zeros(self.n_points, np.int64)
+        c = np.zeros(self.n_points, np.int32)
+        _check(self.lib, self.lib.hx_sim_point_sums(self.h, _p(a), _p(b), _p(c), self.n_points))
+        return a, b, c
 
     def records(self, rec_index: int) -> dict:
         t = self.record_sims[rec_index] // self.n_points

@@ -36,6 +36,7 @@ STAGE_E = 3  # evaluation
 
 POLICY_PQ = 0    # local queue: urgency priority queue (Sec. 4.2)
 POLICY_FCFS = 1  # local queue: first come first served (ablation, Sec. 5.1)
+POLICY_LLF = 2   # local queue: least laxity first, no per-request budget (baseline, Sec. 5.1)
 DISPATCH_WB = 0  # global dispatch: workload balanced (Sec. 4.1)
 DISPATCH_RR = 1  # global dispatch: round robin (ablation, Sec. 5.1)
 
@@ -114,7 +115,7 @@ class Grid:
     gamma_fp: np.ndarray         # int64 [P]  urgency ageing weight * SCALE
     rho: np.ndarray              # int32 [P]  assumed remaining corrections bound
     beta_us2: np.ndarray         # int64 [P]  beta = C_ref * Q_ref, microseconds^2
-    local_policy: np.ndarray     # uint8 [P]  POLICY_PQ / POLICY_FCFS
+    local_policy: np.ndarray     # uint8 [P]  POLICY_PQ / POLICY_FCFS / POLICY_LLF
     dispatch_policy: np.ndarray  # uint8 [P]  DISPATCH_WB / DISPATCH_RR
 
     @property

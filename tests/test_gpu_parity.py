@@ -140,7 +140,8 @@ def test_reduced_recipes_every_sim(cfg, nt, nq, nrec):
 
 
 @pytest.mark.parametrize("local,dispatch", [(W.POLICY_FCFS, W.DISPATCH_WB), (W.POLICY_PQ, W.DISPATCH_RR),
-                                            (W.POLICY_FCFS, W.DISPATCH_RR)])
+                                            (W.POLICY_FCFS, W.DISPATCH_RR), (W.POLICY_LLF, W.DISPATCH_WB),
+                                            (W.POLICY_LLF, W.DISPATCH_RR)])
 def test_policy_variants(local, dispatch):
     wl = W.make_workload(1, n_traces=2, n_queries=300)
     g0 = wl.grid
@@ -278,3 +279,23 @@ def test_full_size_ceiling_sampled():
         bp, bs, _, bper = sim.best(obj)
         assert (bp, bs) == (gp, gs) and bper.tolist() == per.tolist()
     sim.close()
+
+
+def test_point_sums_and_best_of_sums():
+    """Traces split over two handles (as over two ranks): the per-point sums
+    add up to one handle's, and the best point of the sums is its best."""
+    wl = W.make_workload(3, n_traces=4, n_queries=400)
+    wl.grid = W.subset_grid(wl.grid, list(range(0, 512, 3)))
+    whole = gpu(wl)
+    halves = [gpu(W.Workload("h", wl.traces[i:i + 2], wl.cluster, wl.grid, wl.objective)) for i in (0, 2)]
+    sums = [h.point_sums() for h in halves]
+    tot = [sums[0][k] + sums[1][k] for k in range(3)]
+    ref = whole.point_sums()
+    for k in range(3):
+        assert np.array_equal(tot[k], ref[k])
+    nq = sum(t.n_queries for t in wl.traces)
+    for obj in (W.OBJ_P95, W.OBJ_P95_SLO95):
+        bp, bs, bslo, _ = whole.best(obj)
+        assert H.best_of_sums(tot[0], tot[1], tot[2], nq, obj) == (bp, bs, bslo)
+    for h in [whole] + halves:
+        h.close()

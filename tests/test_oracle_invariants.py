@@ -70,12 +70,17 @@ def check_schedule(tr, cl, res, log):
         assert int(res["p95_us"]) == int(np.sort(lat)[rank - 1])
         assert int(res["slo_met"]) == int(np.sum(lat <= p["t_slo"]))
         assert int(res["makespan_us"]) == int(end.max())
+    gold, mixc, m64 = 0x9E3779B97F4A7C15, 0xBF58476D1CE4E5B9, (1 << 64) - 1
+
+    def term(t, idtag):
+        y = ((((t * gold) & m64) ^ idtag) * mixc) & m64
+        return y ^ (y >> 32)
+
     dig = 0
-    gold, m64 = 0x9E3779B97F4A7C15, (1 << 64) - 1
     for c in range(tr.n_calls):
-        dig += _mix64(((int(start[c]) * gold) & m64) ^ ((c << 8) | int(inst[c])))
+        dig += term(int(start[c]), (c << 8) | int(inst[c]))
     for i in range(n):
-        dig += _mix64(((int(end[tr.call_base[i + 1] - 1]) * gold) & m64) ^ ((i << 8) | 0xFF))
+        dig += term(int(end[tr.call_base[i + 1] - 1]), (i << 8) | 0xFF)
     assert dig % (1 << 64) == int(res["digest"])
 
 
@@ -99,7 +104,8 @@ def test_invariants_pq_wb(cfg, nt, nq, points):
 
 
 @pytest.mark.parametrize("local,dispatch", [(W.POLICY_FCFS, W.DISPATCH_WB), (W.POLICY_PQ, W.DISPATCH_RR),
-                                            (W.POLICY_FCFS, W.DISPATCH_RR)])
+                                            (W.POLICY_FCFS, W.DISPATCH_RR), (W.POLICY_LLF, W.DISPATCH_WB),
+                                            (W.POLICY_LLF, W.DISPATCH_RR)])
 def test_invariants_policies(local, dispatch):
     wl = W.make_workload(1, n_traces=1, n_queries=200)
     tr = wl.traces[0]
