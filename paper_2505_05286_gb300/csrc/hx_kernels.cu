@@ -511,7 +511,6 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         if (lane == 0) {
           W->slot[sb + sl] = kKeyInf;
           W->freem[m] |= 1u << sl;
-          W->events++;
         }
         __syncwarp();
         // earliest remaining (end, rid) on m: lanes over its slots
@@ -724,7 +723,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
       hx_result res;
       res.p95_us = st == HX_OK ? (nq > 0 ? W->topk[0] : 0) : -1;
       res.makespan_us = W->makespan;
-      res.events = W->events;
+      res.events = (nc + nq + 8 - steps_left) - qa;
       res.digest = W->digest;
       res.slo_met = W->slo_met;
       res.n_done = n_done;
