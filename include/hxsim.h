@@ -126,6 +126,8 @@ typedef struct hx_options {
   const int32_t* record_sims;       /* [n_record] sim indices (trace * P + point) */
   int32_t max_resident_warps;       /* 0 = fill the GPU */
   int32_t timing;                   /* 1 = time each kernel with CUDA events */
+  int32_t force_generic;            /* 1 = always use the simulation kernel built for
+                                       mixed policies and logging (testing) */
 } hx_options;
 
 /* Per-simulation result, index sim = trace * n_points + point. */

@@ -86,6 +86,7 @@ struct hx_sim {
   std::vector<int32_t> record_sims;
   // launch shape
   int blocks = 0, resident_warps = 0, smem_per_block = 0;
+  bool generic = true;  // which instantiation of the simulation kernel runs
   int64_t scratch_bytes = 0, device_bytes = 0;
   cudaStream_t last_stream = nullptr;
   bool ran = false;
@@ -363,16 +364,22 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
       (rc = upload(h->d_dp, grid->dispatch_policy, h->n_points, s0)))
     return bail(rc);
 
+  // the lean instantiation serves grids that are all workload-balanced
+  // dispatch with the urgency queue and log nothing
+  h->generic = (opt && (opt->n_record > 0 || opt->force_generic));
+  for (int p = 0; p < grid->n_points && !h->generic; ++p)
+    if (grid->local_policy[p] != HX_LOCAL_PQ || grid->dispatch_policy[p] != HX_DISPATCH_WB) h->generic = true;
+  const void* kfn = h->generic ? (const void*)hx::hx_sim_kernel : (const void*)hx::hx_sim_kernel_lean;
   // launch shape of the simulation kernel and its per-warp scratch
   h->smem_per_block = hx::kWarpsPerBlock * ck.smem_per_warp;
-  if (cudaFuncSetAttribute(hx::hx_sim_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, h->smem_per_block) !=
-      cudaSuccess) {
+  if (cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, h->smem_per_block) != cudaSuccess) {
     cudaGetLastError();
     return bail(fail(HX_ERR_CUDA, "cannot reserve shared memory for the simulation kernel"));
   }
   int bps = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, hx::hx_sim_kernel, hx::kWarpsPerBlock * 32,
-                                                    h->smem_per_block) != cudaSuccess || bps < 1) {
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, kfn, hx::kWarpsPerBlock * 32, h->smem_per_block) !=
+          cudaSuccess ||
+      bps < 1) {
     cudaGetLastError();
     return bail(fail(HX_ERR_CUDA, "simulation kernel does not fit on an SM"));
   }
@@ -508,7 +515,10 @@ int hx_sim_run(hx_sim* h, void* stream) {
   hx::hx_prep_kernel<<<prep_blocks, 256, 0, s>>>(pa, h->ck);
   HX_CUDA(cudaGetLastError());
   if (h->timing) HX_CUDA(cudaEventRecord(h->ev[1], s));
-  hx::hx_sim_kernel<<<h->blocks, hx::kWarpsPerBlock * 32, h->smem_per_block, s>>>(sa, h->ck);
+  if (h->generic)
+    hx::hx_sim_kernel<<<h->blocks, hx::kWarpsPerBlock * 32, h->smem_per_block, s>>>(sa, h->ck);
+  else
+    hx::hx_sim_kernel_lean<<<h->blocks, hx::kWarpsPerBlock * 32, h->smem_per_block, s>>>(sa, h->ck);
   HX_CUDA(cudaGetLastError());
   if (h->timing) HX_CUDA(cudaEventRecord(h->ev[2], s));
   hx::hx_best_kernel<<<h->n_traces + 1, 256, 0, s>>>(ba);

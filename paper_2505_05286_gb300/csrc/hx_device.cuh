@@ -26,6 +26,7 @@ constexpr int64_t kTimeInf = INT64_MAX;
 constexpr int kWarpsPerBlock = 4;
 constexpr unsigned kFull = 0xffffffffu;
 constexpr uint64_t kArrivalTag = 64;      // event-key tag: after every instance
+constexpr int kFRows = 18;                // S, G/C with 0..15 corrections done, E
 
 // One call as the simulator reads it: 64 bytes, 16-byte aligned.
 struct __align__(16) CallRec {
@@ -36,7 +37,8 @@ struct __align__(16) CallRec {
   int32_t tbar;       // mean of est over the instances
   int32_t next;       // S: unused; G/C: next correction's id, or ~(E's id) at chain end
   int32_t qid;        // query index within the trace
-  uint8_t stage, u, k, pad;  // stage, corrections done incl. this call, k of the query
+  uint8_t stage, u, k, fcode;  // stage, corrections done incl. this call, k of the query,
+                               // row of the rest-of-path table: S 0, G/C 1 + u, E 17
 };
 static_assert(sizeof(CallRec) == 64, "CallRec is one 64-byte unit");
 
@@ -121,8 +123,9 @@ struct WarpShared {
   uint32_t freem[HX_MAX_INST];  // free-slot mask
   int32_t nslot[HX_MAX_INST];   // slot holding nkey
   // per-simulation constants
-  int64_t A, one_minus_a, G, beta, f_s, f_g, cref_c, cref_e;
-  int32_t rho, rmax, lpol, dpol, recj, kcap, rr, bump;
+  int64_t A, one_minus_a, G, beta;
+  int64_t frest[kFRows];        // rest-of-path cost of the budget denominator by fcode
+  int32_t lpol, dpol, recj, kcap, rr, bump;
   // this warp's scratch slices and the current trace's offsets
   HeapEnt* arena;
   uint8_t* chains;
@@ -154,7 +157,11 @@ struct BestArgs {
 };
 
 __global__ void hx_prep_kernel(PrepArgs a, ClusterK c);
+// hx_sim_kernel: any mix of dispatch and local-queue policies and per-call
+// logs; hx_sim_kernel_lean: every point workload-balanced with the urgency
+// queue, nothing logged (the same simulation with those branches removed).
 __global__ void hx_sim_kernel(SimArgs a, ClusterK c);
+__global__ void hx_sim_kernel_lean(SimArgs a, ClusterK c);
 __global__ void hx_best_kernel(BestArgs a);
 __global__ void hx_selftest_div_kernel(const uint64_t* n, const uint64_t* d, uint64_t* q, uint64_t* q_ref,
                                        int64_t count);

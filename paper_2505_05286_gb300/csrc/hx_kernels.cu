@@ -175,12 +175,13 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
     r.qid = qid;
     r.stage = (uint8_t)st;
     r.k = (uint8_t)k;
-    r.pad = 0;
     if (st == HX_STAGE_S) {
       r.u = 0;
+      r.fcode = 0;
       r.next = -1;
     } else if (st == HX_STAGE_E) {
       r.u = 0;
+      r.fcode = kFRows - 1;
       r.next = -1;
     } else {
       const int cd = a.cand[j];
@@ -193,6 +194,7 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
         nx = (j + 1 < e - 1 && a.stage[j + 1] == HX_STAGE_C && a.cand[j + 1] == cd) ? (int32_t)(j + 1 - cbase) : -1;
       }
       r.next = nx >= 0 ? nx : ~e_rid;
+      r.fcode = (uint8_t)(1 + r.u);
     }
     const int4* src = reinterpret_cast<const int4*>(&r);
     int4* dst = reinterpret_cast<int4*>(a.rec + j);
@@ -374,7 +376,8 @@ __device__ __noinline__ int64_t budget_wide(int64_t num, int64_t tb, int64_t d) 
 #define HX_SIM_MIN_BLOCKS 7
 #endif
 // Resident blocks per SM the register allocation aims for (4 warps each).
-__global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim_kernel(SimArgs a, ClusterK c) {
+template <bool kGeneric>
+__device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -423,27 +426,35 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
       W->nslot[m] = -1;
     }
     for (int j = lane; j < c.total_slots; j += 32) W->slot[j] = kKeyInf;
-    if (lane == 0) {
-      // stage reference costs: mean over instances of Eq. (comp) at the stage's reference tokens
+    if (lane < kFRows) {
+      // rest of the request's own path after it (the budget denominator minus
+      // its own mean cost): stage reference costs, i.e. means over instances of
+      // Eq. (comp) at the stage's reference tokens, for G, min(rho, R - u)
+      // corrections and E
       int64_t cref[4];
       for (int s = 0; s < 4; ++s) {
         int64_t sum = 0;
         for (int ty = 0; ty < c.n_types; ++ty) sum += cost_on_type(c, ty, c.ref_prompt[s], c.ref_out[s]) * c.cnt[ty];
         cref[s] = sum / N;
       }
-      const int64_t A = a.alpha[p], rho = a.rho[p], rmax = c.rmax;
-      const int64_t corr_plan = rho < rmax ? rho : rmax;
+      const int64_t rho = a.rho[p], rmax = c.rmax;
+      int64_t f;
+      if (lane == 0) {
+        f = cref[HX_STAGE_G] + (rho < rmax ? rho : rmax) * cref[HX_STAGE_C] + cref[HX_STAGE_E];
+      } else if (lane == kFRows - 1) {
+        f = 0;
+      } else {
+        const int64_t left = rmax - (lane - 1);
+        f = (rho < left ? rho : left) * cref[HX_STAGE_C] + cref[HX_STAGE_E];
+      }
+      W->frest[lane] = f;
+    }
+    if (lane == 0) {
+      const int64_t A = a.alpha[p];
       W->A = A;
       W->one_minus_a = kScale - A;
       W->G = a.gamma[p];
       W->beta = a.beta[p];
-      // rest-of-path costs of the budget denominator for S and G calls
-      W->f_s = cref[HX_STAGE_G] + corr_plan * cref[HX_STAGE_C] + cref[HX_STAGE_E];
-      W->f_g = corr_plan * cref[HX_STAGE_C] + cref[HX_STAGE_E];
-      W->cref_c = cref[HX_STAGE_C];
-      W->cref_e = cref[HX_STAGE_E];
-      W->rho = (int32_t)rho;
-      W->rmax = (int32_t)rmax;
       W->lpol = a.lpol[p];
       W->dpol = a.dpol[p];
       W->recj = a.rec_map ? a.rec_map[sim] : -1;
@@ -574,16 +585,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         const int64_t dl = r->deadline;
         const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
         const int64_t tb = tail.x;
-        const int stg = tail.w & 0xff;
-        int64_t f;
-        if (stg == HX_STAGE_S) f = W->f_s;
-        else if (stg == HX_STAGE_G) f = W->f_g;
-        else if (stg == HX_STAGE_C) {
-          const int64_t left = (int64_t)W->rmax - ((tail.w >> 8) & 0xff);
-          const int64_t rho = W->rho;
-          f = (rho < left ? rho : left) * W->cref_c + W->cref_e;
-        } else f = 0;
-        const int64_t dd = tb + f;
+        const int64_t dd = tb + W->frest[(uint32_t)tail.w >> 24];
         const int64_t num = dl - now;
         const bool small = num > -(int64_t(1) << 34) && num < (int64_t(1) << 34);
         // SIMT division passes: each lane refreshes one stale reward of its
@@ -593,7 +595,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         bool need_budget = small;
         int bl = 0;
         const uint64_t beta = (uint64_t)W->beta;
-        if (W->one_minus_a == 0 || W->dpol == HX_DISPATCH_RR) {
+        if (W->one_minus_a == 0 || (kGeneric && W->dpol == HX_DISPATCH_RR)) {
           // rewards carry no weight at alpha = 1 and are unused by round robin
           dirty0 = false;
           dirty1 = false;
@@ -616,7 +618,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         }
         const int64_t budget = small ? __shfl_sync(kFull, bres, bl) : budget_wide(num, tb, dd);
         int m;
-        if (W->dpol == HX_DISPATCH_RR) {
+        if (kGeneric && W->dpol == HX_DISPATCH_RR) {
           m = W->rr;
           __syncwarp();
           if (lane == 0) W->rr = (m + 1 == N) ? 0 : m + 1;
@@ -638,7 +640,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         // local-queue key, higher first: Eq. (priority) aged by gamma with the
         // common now dropped; FCFS: earliest enqueue; LLF: least deadline - now -
         // remaining work, again with the common now dropped
-        const int lpol = W->lpol;
+        const int lpol = kGeneric ? W->lpol : HX_LOCAL_PQ;
         const long long key = lpol == HX_LOCAL_PQ     ? (long long)(kScale * (est_m - budget) - W->G * now)
                               : lpol == HX_LOCAL_FCFS ? (long long)(-now)
                                                       : (long long)(dd - dl);
@@ -650,8 +652,10 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
         }
         npend++;
         touched |= 1ull << m;
-        const int recj = W->recj;
-        if (recj >= 0 && lane == 0) log_dispatch(a, recj, rid, m, now, budget);
+        if (kGeneric) {
+          const int recj = W->recj;
+          if (recj >= 0 && lane == 0) log_dispatch(a, recj, rid, m, now, budget);
+        }
       }
 
       // Batch boundary on every touched instance: its free slots go to the most
@@ -705,8 +709,10 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
               W->nslot[m] = sl;
             }
             W->digest += call_term(rid, m, now);
-            const int recj = W->recj;
-            if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
+            if (kGeneric) {
+              const int recj = W->recj;
+              if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
+            }
           }
           __syncwarp();
         }
@@ -734,6 +740,14 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim
     }
     __syncwarp();
   }
+}
+
+__global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim_kernel(SimArgs a, ClusterK c) {
+  sim_body<true>(a, c);
+}
+
+__global__ void __launch_bounds__(kWarpsPerBlock * 32, HX_SIM_MIN_BLOCKS) hx_sim_kernel_lean(SimArgs a, ClusterK c) {
+  sim_body<false>(a, c);
 }
 
 // ---------------------------------------------------------- best kernel

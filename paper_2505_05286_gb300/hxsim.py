@@ -59,7 +59,8 @@ class hx_grid(ctypes.Structure):
 
 class hx_options(ctypes.Structure):
     _fields_ = [("n_record", ctypes.c_int32), ("record_sims", ctypes.c_void_p),
-                ("max_resident_warps", ctypes.c_int32), ("timing", ctypes.c_int32)]
+                ("max_resident_warps", ctypes.c_int32), ("timing", ctypes.c_int32),
+                ("force_generic", ctypes.c_int32)]
 
 
 class hx_best(ctypes.Structure):
@@ -204,7 +205,7 @@ class Sim:
     """A set of (trace x point) simulations resident on the current CUDA device."""
 
     def __init__(self, traces, cluster, grid, record_sims: Sequence[int] = (), timing: bool = False,
-                 max_resident_warps: int = 0):
+                 max_resident_warps: int = 0, force_generic: bool = False):
         self.lib = load()
         self.n_traces = len(traces)
         self.n_points = int(grid.alpha_fp.shape[0])
@@ -222,7 +223,8 @@ class Sim:
         hg = hx_grid(self.n_points, *[_p(x) for x in gcols])
         self.record_sims = [int(s) for s in record_sims]
         rs = _c(self.record_sims if self.record_sims else [0], np.int32)
-        opt = hx_options(len(self.record_sims), _p(rs), int(max_resident_warps), int(bool(timing)))
+        opt = hx_options(len(self.record_sims), _p(rs), int(max_resident_warps), int(bool(timing)),
+                         int(bool(force_generic)))
         h = ctypes.c_void_p()
         _check(self.lib, self.lib.hx_sim_create(tr.arr, self.n_traces, ctypes.byref(hc), ctypes.byref(hg),
                                                 ctypes.byref(opt), ctypes.byref(h)))

@@ -177,7 +177,7 @@ def stream_uniform(key: int, n: int, start: int = 0) -> np.ndarray:
     return (stream_u64(key, n, start) >> np.uint64(11)).astype(np.float64) * (2.0 ** -53)
 
 
-_STREAM_ARRIVAL, _STREAM_DWELL, _STREAM_K, _STREAM_ERR, _STREAM_PROMPT, _STREAM_OUT = range(1, 7)
+_STREAM_ARRIVAL, _STREAM_DWELL, _STREAM_K, _STREAM_ERR, _STREAM_PROMPT, _STREAM_OUT, _STREAM_EST = range(1, 8)
 
 
 # ----------------------------------------------------------------------------
@@ -218,6 +218,7 @@ class Recipe:
     c_ref_us: int                # reference computation / queueing time (beta = c_ref^2)
     objective: int
     trace_seeds: Optional[Sequence[int]] = None
+    est_noise_sigma: float = 0.0  # lognormal noise of the believed output length (0: the stage mean)
 
 
 def _u(a, b):
@@ -270,6 +271,22 @@ CONFIGS: List[Recipe] = [
            TYPES_4, [26, 19, 13, 6], 2, 5 * SCALE // 2,
            8, _GAMMA8, [0, 1, 2, 3], [(1, 4), (1, 2), (1, 1), (2, 1)], 500_000, OBJ_P95_SLO95),
 ]
+
+# Extra recipes beyond the five benchmark ones (Sec. 5.1's workload shapes):
+#  - "paper-shaped": ~20 calls per query (k = 8 candidates, error probability
+#    0.55, up to 10 refinement rounds) at 1 query/s on a 2A + 2B cluster;
+#  - "noisy-estimate": recipe 1 with the output-length predictor replaced by
+#    the true length times lognormal(0, 0.5) noise.
+EXTRA: dict = {
+    "paper-shaped": Recipe("paper-shaped-8x400q-4inst-16pt", 8, 400, "poisson", [1.0], 0.0, [8, 8], 0.55, 10,
+                           _UNIF_PROMPT, _UNIF_OUT, _UNIF_OUT_EST, _UNIF_REF_PROMPT,
+                           [TYPE_A, TYPE_B], [2, 2], 0, 3 * SCALE,
+                           4, _GAMMA4, None, [(1, 1)], 400_000, OBJ_P95),
+    "noisy-estimate": Recipe("noisy-estimate-8x2000q-8inst-64pt", 8, 2000, "poisson", [4.0], 0.0, [4, 4], 0.3, 2,
+                             _UNIF_PROMPT, _UNIF_OUT, _UNIF_OUT_EST, _UNIF_REF_PROMPT,
+                             [TYPE_A, TYPE_B, TYPE_C], [4, 2, 2], 0, 3 * SCALE,
+                             8, _GAMMA8, None, [(1, 1)], 300_000, OBJ_P95, est_noise_sigma=0.5),
+}
 
 
 # ----------------------------------------------------------------------------
@@ -403,6 +420,12 @@ def make_trace(recipe: Recipe, cfg_id: int, seed: int, n_queries: Optional[int] 
     prompt = _draw_tokens(stream_key(key, _STREAM_PROMPT), stage, recipe.prompt)
     out = _draw_tokens(stream_key(key, _STREAM_OUT), stage, recipe.out)
     out_est = np.asarray(recipe.out_est, dtype=np.int32)[stage]
+    if recipe.est_noise_sigma > 0:
+        # an output-length predictor with multiplicative lognormal error around the truth
+        ue = stream_uniform(stream_key(key, _STREAM_EST), 2 * nc).reshape(nc, 2)
+        z = np.sqrt(-2.0 * np.log(1.0 - ue[:, 0])) * np.cos(2.0 * np.pi * ue[:, 1])
+        est = np.floor(out.astype(np.float64) * np.exp(recipe.est_noise_sigma * z) + 0.5)
+        out_est = np.clip(est, 0, 1 << 20).astype(np.int32)
     return Trace(arrival.astype(np.int64), k.astype(np.uint8), call_base.astype(np.int32),
                  prompt, out, out_est.astype(np.int32), stage, cand, retry)
 
@@ -431,10 +454,13 @@ def make_grid(recipe: Recipe, local_policy: int = POLICY_PQ, dispatch_policy: in
                 np.full(P, dispatch_policy, np.uint8))
 
 
-def make_workload(cfg_id: int, n_traces: Optional[int] = None, n_queries: Optional[int] = None,
+def make_workload(cfg_id, n_traces: Optional[int] = None, n_queries: Optional[int] = None,
                   first_trace: int = 0) -> Workload:
-    """Workload of recipe `cfg_id`, optionally with fewer traces or queries."""
-    r = CONFIGS[cfg_id]
+    """Workload of recipe `cfg_id` (an index of CONFIGS or a key of EXTRA),
+    optionally with fewer traces or queries."""
+    r = CONFIGS[cfg_id] if isinstance(cfg_id, int) else EXTRA[cfg_id]
+    if not isinstance(cfg_id, int):
+        cfg_id = 16 + sorted(EXTRA).index(cfg_id)
     nt = r.n_traces if n_traces is None else int(n_traces)
     traces = [make_trace(r, cfg_id, first_trace + j, n_queries) for j in range(nt)]
     name = r.name if (n_traces is None and n_queries is None) else (

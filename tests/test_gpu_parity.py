@@ -299,3 +299,30 @@ def test_point_sums_and_best_of_sums():
         assert H.best_of_sums(tot[0], tot[1], tot[2], nq, obj) == (bp, bs, bslo)
     for h in [whole] + halves:
         h.close()
+
+
+@pytest.mark.parametrize("name,nt,nq", [("paper-shaped", 3, 150), ("noisy-estimate", 2, 300)])
+def test_extra_recipes_every_sim(name, nt, nq):
+    """~20 calls per query with up to 10 refinement rounds, and a noisy
+    output-length estimate: every simulation and two full logs."""
+    wl = W.make_workload(name, n_traces=nt, n_queries=nq)
+    sim = gpu(wl, record=[1, wl.n_sims - 2])
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(sim.results(), o, name)
+    assert_logs(sim, wl, 0)
+    assert_logs(sim, wl, 1)
+    check_best(sim, wl, o)
+    sim.close()
+
+
+def test_lean_and_generic_kernels_agree():
+    """The simulation kernel built for uniform WB + urgency-queue grids without
+    logs gives exactly what the general one gives."""
+    wl = W.make_workload(4, n_traces=2, n_queries=400)
+    lean = gpu(wl)
+    full = gpu(wl, force_generic=True)
+    assert_same(lean.results(), full.results(), "lean vs generic")
+    o = oracle_results(wl, list(range(0, wl.n_sims, 37)) + [wl.n_sims - 1])
+    assert_same(lean.results()[list(range(0, wl.n_sims, 37)) + [wl.n_sims - 1]], o, "lean vs oracle")
+    lean.close()
+    full.close()

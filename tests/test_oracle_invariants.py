@@ -151,3 +151,13 @@ def test_rejects_malformed():
     pt = oracle.point_of(wl.grid, 0)
     pt["alpha_fp"] = W.SCALE + 1
     assert oracle.simulate(tr, wl.cluster, pt)["status"] == 1
+
+
+@pytest.mark.parametrize("name", ["paper-shaped", "noisy-estimate"])
+def test_invariants_extra_recipes(name):
+    wl = W.make_workload(name, n_traces=1, n_queries=120)
+    tr = wl.traces[0]
+    for p in [0, wl.grid.n_points // 2, wl.grid.n_points - 1]:
+        res, log = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, p), check=True, log=True)
+        assert res["status"] == 0
+        check_schedule(tr, wl.cluster, res, log)
