@@ -208,10 +208,6 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
 // -------------------------------------------------------- simulation kernel
 namespace {
 
-__device__ __forceinline__ int pick4(const int4& v, int t) {
-  return t == 0 ? v.x : (t == 1 ? v.y : (t == 2 ? v.z : v.w));
-}
-
 __device__ __forceinline__ bool ent_better(long long ka, int ra, long long kb, int rb) {
   return ka > kb || (ka == kb && ra < rb);
 }
@@ -580,8 +576,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       for (int32_t jr = 0; jr < rel_count; ++jr) {
         const int32_t rid = rel_first + jr;
         const CallRec* r = rec + rid;
-        const int4 e4 = *reinterpret_cast<const int4*>(r->est);
-        const int4 s4 = *reinterpret_cast<const int4*>(r->svc);
+        // Eq. (comp) and the service time on this lane's two instances
+        const int e0 = r->est[ty0], e1 = r->est[ty1];
+        const int v0 = r->svc[ty0], v1 = r->svc[ty1];
         const int64_t dl = r->deadline;
         const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
         const int64_t tb = tail.x;
@@ -624,14 +621,14 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           if (lane == 0) W->rr = (m + 1 == N) ? 0 : m + 1;
         } else {
           const int64_t A = W->A, oma = W->one_minus_a;
-          const int64_t s0 = valid0 ? oma * rew0 - A * (int64_t)pick4(e4, ty0) : INT64_MIN;
-          const int64_t s1 = valid1 ? oma * rew1 - A * (int64_t)pick4(e4, ty1) : INT64_MIN;
+          const int64_t s0 = valid0 ? oma * rew0 - A * (int64_t)e0 : INT64_MIN;
+          const int64_t s1 = valid1 ? oma * rew1 - A * (int64_t)e1 : INT64_MIN;
           const bool take1 = s1 > s0;
           m = warp_argmax_s64(take1 ? s1 : s0, take1 ? m1 : m0);
         }
-        const int tym = c.inst_type[m];
-        const int64_t est_m = pick4(e4, tym);
-        const int svc_m = pick4(s4, tym);
+        // the winner's costs, from the lane that owns it
+        const int64_t est_m = __shfl_sync(kFull, m < 32 ? e0 : e1, m & 31);
+        const int svc_m = __shfl_sync(kFull, m < 32 ? v0 : v1, m & 31);
         if (lane == (m & 31)) {
           W->q[m] += est_m;
           if (m < 32) dirty0 = true;
