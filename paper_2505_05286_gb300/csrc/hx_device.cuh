@@ -113,15 +113,15 @@ struct SimArgs {
 
 // Per-warp shared memory of one simulation: per-instance local-queue and
 // slot state, per-simulation constants and lane-0 accumulators, then one
-// 64-bit (end << 24 | request id) key per batch slot of the cluster.
+// 64-bit (end << 24 | request id) key per batch slot of the cluster.  An
+// instance's running calls occupy the first cnt of its slots in ascending key
+// order, so the next completion on it is always its first slot.
 struct WarpShared {
   int64_t q[HX_MAX_INST];       // t_queue: Eq. comp summed over requests dispatched and unfinished
-  uint64_t nkey[HX_MAX_INST];   // earliest running (end << 24 | rid), or all ones
   int32_t hoff[HX_MAX_INST];    // local queue: heap offset in the arena
   int32_t hcap[HX_MAX_INST];    //              heap capacity
   int32_t hsize[HX_MAX_INST];   //              heap size
-  uint32_t freem[HX_MAX_INST];  // free-slot mask
-  int32_t nslot[HX_MAX_INST];   // slot holding nkey
+  int32_t cnt[HX_MAX_INST];     // running calls (the first cnt of the instance's slot keys)
   // per-simulation constants
   int64_t A, one_minus_a, G, beta;
   int64_t frest[kFRows];        // rest-of-path cost of the budget denominator by fcode

@@ -414,12 +414,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     }
 
     for (int m = lane; m < 64; m += 32) {
-      W->nkey[m] = kKeyInf;
       W->hoff[m] = 0;
       W->hcap[m] = 0;
       W->hsize[m] = 0;
-      W->freem[m] = m < N ? ((1u << c.inst_slots[m]) - 1u) : 0u;
-      W->nslot[m] = -1;
+      W->cnt[m] = 0;
     }
     for (int j = lane; j < c.total_slots; j += 32) W->slot[j] = kKeyInf;
     if (lane < kFRows) {
@@ -506,29 +504,21 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         // completion on instance m
         const int m = (int)(ck & 127ull);
         now = (int64_t)(ck >> 7);
-        const int sb = c.slot_base[m];
-        const int sl = W->nslot[m];
-        const int32_t rid = (int32_t)(W->slot[sb + sl] & 0xffffffull);
-        // the finished call's record: issued now, used after the slot rescan
+        uint64_t* const sl = W->slot + c.slot_base[m];
+        const int cn = W->cnt[m];
+        // the finishing call heads m's sorted slots
+        const int32_t rid = (int32_t)(sl[0] & 0xffffffull);
+        // the finished call's record: issued now, used after the slot shift
         const CallRec* r = rec + rid;
         const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
         const int64_t est_m = r->est[c.inst_type[m]];
         const int hs_m = W->hsize[m];
+        // remove it: the remaining keys move down one slot
+        const uint64_t nxt = lane + 1 < cn ? sl[lane + 1] : kKeyInf;
         __syncwarp();
-        if (lane == 0) {
-          W->slot[sb + sl] = kKeyInf;
-          W->freem[m] |= 1u << sl;
-        }
-        __syncwarp();
-        // earliest remaining (end, rid) on m: lanes over its slots
-        const uint64_t sk = lane < c.inst_slots[m] ? W->slot[sb + lane] : kKeyInf;
-        const uint64_t mk = warp_min_u64(sk);
-        const unsigned who = __ballot_sync(kFull, sk == mk && mk != kKeyInf);
-        if (lane == 0) {
-          W->nkey[m] = mk;
-          W->nslot[m] = who ? __ffs(who) - 1 : -1;
-        }
-        set_key(m, mk);
+        if (lane < cn) sl[lane] = nxt;
+        if (lane == 0) W->cnt[m] = cn - 1;
+        set_key(m, __shfl_sync(kFull, nxt, 0));
         if (lane == (m & 31)) {
           W->q[m] -= est_m;
           if (m < 32) dirty0 = true;
@@ -661,14 +651,14 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       while (tm) {
         const int m = __ffsll((long long)tm) - 1;
         tm &= tm - 1;
-        const uint32_t fm = W->freem[m];
-        const int hs = W->hsize[m];
-        const uint64_t nkey0 = W->nkey[m];
+        uint64_t* const sl = W->slot + c.slot_base[m];
+        const int ns = c.inst_slots[m];
         const unsigned pm = __ballot_sync(kFull, lane < npend && pend_m == m);
         __syncwarp();
-        uint64_t nkey = nkey0;  // lane 0 tracks the instance's earliest (end, rid)
+        int cn = W->cnt[m];
+        const int hs = W->hsize[m];
         // fast path: an empty queue with room for all of this event's arrivals
-        const bool direct = hs == 0 && __popc(pm) <= __popc(fm);
+        const bool direct = hs == 0 && __popc(pm) <= ns - cn;
         if (!direct && pm) {
           status = push_pending(W, W->arena, a.arena_per_warp, m, pm, pend_key, pend_rid, pend_svc, lane);
           if (status != HX_OK) break;
@@ -684,27 +674,21 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             svc = __shfl_sync(kFull, pend_svc, j);
           } else {
             const int n = W->hsize[m];
-            const bool go = W->freem[m] != 0u && n > 0;
             __syncwarp();
-            if (!go) break;
+            if (cn >= ns || n == 0) break;
             const HeapEnt top = heap_pop_warp(W->arena + W->hoff[m], n, lane);
             if (lane == 0) W->hsize[m] = n - 1;
             rid = top.rid;
             svc = top.svc;
           }
+          // run it until now + svc: insert its key into m's sorted slots
+          const uint64_t nk = ((uint64_t)(now + svc) << 24) | (uint64_t)(uint32_t)rid;
+          const uint64_t cur = lane < cn ? sl[lane] : kKeyInf;
+          const int pos = __popc(__ballot_sync(kFull, cur < nk));
+          if (lane >= pos && lane < cn) sl[lane + 1] = cur;
+          if (lane == pos) sl[pos] = nk;
+          ++cn;
           if (lane == 0) {
-            // occupy a free slot until now + svc
-            const int sb = c.slot_base[m];
-            const uint32_t fr = W->freem[m];
-            const int sl = __ffs(fr) - 1;
-            W->freem[m] = fr & ~(1u << sl);
-            const uint64_t nk = ((uint64_t)(now + svc) << 24) | (uint64_t)(uint32_t)rid;
-            W->slot[sb + sl] = nk;
-            if (nk < nkey) {
-              nkey = nk;
-              W->nkey[m] = nk;
-              W->nslot[m] = sl;
-            }
             W->digest += call_term(rid, m, now);
             if (kGeneric) {
               const int recj = W->recj;
@@ -713,7 +697,8 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           }
           __syncwarp();
         }
-        set_key(m, __shfl_sync(kFull, nkey, 0));
+        if (lane == 0) W->cnt[m] = cn;
+        set_key(m, cn ? sl[0] : kKeyInf);
       }
       if (status != HX_OK) break;
     }
