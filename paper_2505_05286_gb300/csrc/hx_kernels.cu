@@ -468,7 +468,12 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     // (t_queue of instance m lives in W->q[m], touched only by its owner lane)
     W->q[m0] = 0;
     W->q[m1] = 0;
-    int64_t rew0 = reward_of(W->beta, 0), rew1 = rew0;
+    // (1 - alpha) * reward per instance; instances past N score far below any
+    // real one (|alpha * est| < 2^52), so the argmax needs no validity test
+    const int32_t oma32 = (int32_t)W->one_minus_a;
+    const int64_t orew_idle = (int64_t)oma32 * reward_of(W->beta, 0);
+    int64_t orew0 = valid0 ? orew_idle : -(int64_t(1) << 62);
+    int64_t orew1 = valid1 ? orew_idle : -(int64_t(1) << 62);
     bool dirty0 = false, dirty1 = false;
     uint64_t k0 = kKeyInf, k1 = kKeyInf;
     // this event's dispatches, entry j on lane j
@@ -587,19 +592,21 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           dirty0 = false;
           dirty1 = false;
         }
+        const uint64_t bn = (uint64_t)(num < 0 ? -num : num) * (uint64_t)tb;
         for (;;) {
-          const unsigned busy = __ballot_sync(kFull, dirty0 || dirty1);
+          const bool rj = dirty0 || dirty1;
+          const unsigned busy = __ballot_sync(kFull, rj);
           const int cand = (need_budget && ~busy) ? __ffs(~busy) - 1 : -1;
-          uint64_t n = 0, d = 1;
-          int job = 0;
-          if (dirty0) { const int64_t q = W->q[m0]; n = beta; d = q > 1 ? q : 1; job = 1; }
-          else if (dirty1) { const int64_t q = W->q[m1]; n = beta; d = q > 1 ? q : 1; job = 2; }
-          else if (lane == cand) { n = (uint64_t)(num < 0 ? -num : num) * (uint64_t)tb; d = (uint64_t)dd; job = 3; }
+          const bool bj = lane == cand;  // never a lane with a stale reward
+          const int64_t q = W->q[dirty0 ? m0 : m1];
+          const uint64_t n = rj ? beta : (bj ? bn : 0);
+          const uint64_t d = rj ? (uint64_t)(q > 1 ? q : 1) : (bj ? (uint64_t)dd : 1);
           const uint64_t res = udiv_trial(n, d);
-          const int64_t capped = res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap;
-          if (job == 1) { rew0 = capped; dirty0 = false; }
-          else if (job == 2) { rew1 = capped; dirty1 = false; }
-          else if (job == 3) { bres = num < 0 ? -(int64_t)res : (int64_t)res; }
+          const int64_t orew =
+              (int64_t)(int32_t)W->one_minus_a * (res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap);
+          if (dirty0) { orew0 = orew; dirty0 = false; }
+          else if (dirty1) { orew1 = orew; dirty1 = false; }
+          if (bj) bres = num < 0 ? -(int64_t)res : (int64_t)res;
           if (cand >= 0) { bl = cand; need_budget = false; }
           if (!need_budget && !__any_sync(kFull, dirty0 || dirty1)) break;
         }
@@ -610,9 +617,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           __syncwarp();
           if (lane == 0) W->rr = (m + 1 == N) ? 0 : m + 1;
         } else {
-          const int64_t A = W->A, oma = W->one_minus_a;
-          const int64_t s0 = valid0 ? oma * rew0 - A * (int64_t)e0 : INT64_MIN;
-          const int64_t s1 = valid1 ? oma * rew1 - A * (int64_t)e1 : INT64_MIN;
+          const int32_t A = (int32_t)W->A;
+          const int64_t s0 = orew0 - (int64_t)A * e0;
+          const int64_t s1 = orew1 - (int64_t)A * e1;
           const bool take1 = s1 > s0;
           m = warp_argmax_s64(take1 ? s1 : s0, take1 ? m1 : m0);
         }
