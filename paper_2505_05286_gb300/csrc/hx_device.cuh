@@ -122,6 +122,9 @@ struct WarpShared {
   int32_t hcap[HX_MAX_INST];    //              heap capacity
   int32_t hsize[HX_MAX_INST];   //              heap size
   int32_t cnt[HX_MAX_INST];     // running calls (the first cnt of the instance's slot keys)
+  // this event's dispatches in order: local-queue key, (request id, service time)
+  int64_t pkey[32];
+  int2 prs[32];
   // per-simulation constants
   int64_t A, one_minus_a, G, beta;
   int64_t frest[kFRows];        // rest-of-path cost of the budget denominator by fcode
@@ -131,7 +134,10 @@ struct WarpShared {
   uint8_t* chains;
   int64_t* topk;
   int64_t qb, cb;
-  int32_t nq, pad0;
+  int32_t nq, nc;
+  int64_t sim, clk0;            // result index and start clock of the simulation
+  uint64_t akey;                // next arrival's event key (written alike by every lane)
+  int32_t qa, pad0;             // arrivals taken so far (likewise)
   // lane-0 accumulators
   uint64_t digest;
   int64_t makespan;

@@ -314,13 +314,13 @@ __device__ __noinline__ void topk_insert(int64_t* h, int& n, int kcap, int64_t v
 // mask pm) in m's heap, re-homing the heap in the arena when it is full.
 // All lanes call.  Returns HX_OK or HX_ERR_CAPACITY.
 __device__ __noinline__ int push_pending(WarpShared* W, HeapEnt* arena, int64_t arena_per_warp, int m, unsigned pm,
-                                        long long pend_key, int pend_rid, int pend_svc, int lane) {
+                                        int lane) {
   while (pm) {
     const int j = __ffs(pm) - 1;
     pm &= pm - 1;
-    const long long key = __shfl_sync(kFull, pend_key, j);
-    const int rid = __shfl_sync(kFull, pend_rid, j);
-    const int svc = __shfl_sync(kFull, pend_svc, j);
+    const long long key = W->pkey[j];
+    const int2 rs = W->prs[j];
+    const int rid = rs.x, svc = rs.y;
     const int size = W->hsize[m], cap = W->hcap[m], off = W->hoff[m], bump = W->bump;
     __syncwarp();
     int hoff = off;
@@ -411,6 +411,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       W->qb = qb;
       W->cb = cb;
       W->nq = nq;
+      W->nc = nc;
+      W->sim = sim;
+      W->clk0 = clk0;
     }
 
     for (int m = lane; m < 64; m += 32) {
@@ -477,11 +480,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     bool dirty0 = false, dirty1 = false;
     uint64_t k0 = kKeyInf, k1 = kKeyInf;
     // this event's dispatches, entry j on lane j
-    int pend_m = -1, pend_rid = 0, pend_svc = 0;
-    long long pend_key = 0;
+    int pend_m = -1;
 
-    int32_t qa = 0;
-    uint64_t akey = nq > 0 ? (((uint64_t)a.arrival[qb] << 7) | kArrivalTag) : kKeyInf;
+    W->qa = 0;
+    W->akey = nq > 0 ? (((uint64_t)a.arrival[qb] << 7) | kArrivalTag) : kKeyInf;
     int64_t now = 0;
     int32_t status = HX_OK, npend = 0;
     uint64_t touched = 0;
@@ -496,6 +498,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
 
     for (;;) {
       const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
+      const uint64_t akey = W->akey;
       if (ck == kKeyInf && akey == kKeyInf) break;
       if (--steps_left < 0) {
         status = HX_ERR_STEP_LIMIT;
@@ -560,10 +563,11 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       } else {
         now = (int64_t)(akey >> 7);
         const int64_t qbase = W->qb;
+        const int32_t qa = W->qa;
         rel_first = (int32_t)(a.qcall[qbase + qa] - W->cb);
         rel_count = 1;
-        qa++;
-        akey = qa < W->nq ? (((uint64_t)a.arrival[qbase + qa] << 7) | kArrivalTag) : kKeyInf;
+        W->qa = qa + 1;
+        W->akey = qa + 1 < W->nq ? (((uint64_t)a.arrival[qbase + qa + 1] << 7) | kArrivalTag) : kKeyInf;
       }
 
       // Sec. 4.1 + 4.2 for each released request, in request-id order: budget at
@@ -640,9 +644,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
                                                       : (long long)(dd - dl);
         if (lane == npend) {
           pend_m = m;
-          pend_key = key;
-          pend_rid = rid;
-          pend_svc = svc_m;
+        }
+        if (lane == 0) {
+          W->pkey[npend] = key;
+          W->prs[npend] = make_int2(rid, svc_m);
         }
         npend++;
         touched |= 1ull << m;
@@ -667,7 +672,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         // fast path: an empty queue with room for all of this event's arrivals
         const bool direct = hs == 0 && __popc(pm) <= ns - cn;
         if (!direct && pm) {
-          status = push_pending(W, W->arena, a.arena_per_warp, m, pm, pend_key, pend_rid, pend_svc, lane);
+          status = push_pending(W, W->arena, a.arena_per_warp, m, pm, lane);
           if (status != HX_OK) break;
         }
         unsigned bits = direct ? pm : 0u;
@@ -677,8 +682,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             if (!bits) break;
             const int j = __ffs(bits) - 1;
             bits &= bits - 1;
-            rid = __shfl_sync(kFull, pend_rid, j);
-            svc = __shfl_sync(kFull, pend_svc, j);
+            const int2 rs = W->prs[j];
+            rid = rs.x;
+            svc = rs.y;
           } else {
             const int n = W->hsize[m];
             __syncwarp();
@@ -718,14 +724,14 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       hx_result res;
       res.p95_us = st == HX_OK ? (nq > 0 ? W->topk[0] : 0) : -1;
       res.makespan_us = W->makespan;
-      res.events = (nc + nq + 8 - steps_left) - qa;
+      res.events = (W->nc + nq + 8 - steps_left) - W->qa;
       res.digest = W->digest;
       res.slo_met = W->slo_met;
       res.n_done = n_done;
       res.status = st;
-      const long long dc = (clock64() - clk0) >> 10;
+      const long long dc = (clock64() - W->clk0) >> 10;
       res.cycles_k = dc < INT32_MAX ? (int32_t)dc : INT32_MAX;
-      a.results[sim] = res;
+      a.results[W->sim] = res;
     }
     __syncwarp();
   }
