@@ -142,6 +142,10 @@ struct WarpShared {
   uint64_t digest;
   int64_t makespan;
   int32_t n_done, slo_met, events, tk;
+  int64_t tkmin;                // root of the full top-K heap (written alike by every lane)
+  int64_t dt[32];               // digest terms waiting to be hashed: time, id tag
+  uint32_t dtag[32];
+  int32_t dn, pad1;             // terms waiting (written alike by every lane)
   uint64_t slot[1];             // [total_slots]
 };
 

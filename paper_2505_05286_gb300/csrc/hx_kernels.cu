@@ -25,13 +25,9 @@ __device__ __forceinline__ uint64_t digest_term(uint64_t t, uint64_t idtag) {
   return y ^ (y >> 32);
 }
 
-__device__ __forceinline__ uint64_t call_term(int32_t rid, int inst, int64_t start) {
-  return digest_term((uint64_t)start, ((uint64_t)(uint32_t)rid << 8) | (uint64_t)inst);
-}
-
-__device__ __forceinline__ uint64_t query_term(int32_t qid, int64_t end) {
-  return digest_term((uint64_t)end, ((uint64_t)(uint32_t)qid << 8) | 0xFFull);
-}
+// Id tags: a call's start is (rid << 8 | instance), a query's end (qid << 8 | 0xFF).
+__device__ __forceinline__ uint32_t call_tag(int32_t rid, int inst) { return ((uint32_t)rid << 8) | (uint32_t)inst; }
+__device__ __forceinline__ uint32_t query_tag(int32_t qid) { return ((uint32_t)qid << 8) | 0xFFu; }
 
 __device__ __forceinline__ uint64_t warp_min_u64(uint64_t v) {
   uint32_t hi = (uint32_t)(v >> 32), lo = (uint32_t)v;
@@ -208,6 +204,29 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
 // -------------------------------------------------------- simulation kernel
 namespace {
 
+// The digest is a sum of terms, so they are hashed 32 at a time: every lane
+// calls with the same (t, tag); lane 0 appends it, and a full batch is hashed
+// one term per lane and summed into W->digest.
+__device__ __noinline__ void digest_flush(WarpShared* W, int n, int lane) {
+  __syncwarp();
+  uint64_t y = lane < n ? digest_term((uint64_t)W->dt[lane], W->dtag[lane]) : 0ull;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) y += __shfl_xor_sync(kFull, y, o);
+  if (lane == 0) W->digest += y;
+  W->dn = 0;
+  __syncwarp();
+}
+
+__device__ __forceinline__ void digest_push(WarpShared* W, int64_t t, uint32_t tag, int lane) {
+  const int n = W->dn;
+  if (lane == 0) {
+    W->dt[n] = t;
+    W->dtag[n] = tag;
+  }
+  if (n == 31) digest_flush(W, 32, lane);
+  else W->dn = n + 1;
+}
+
 __device__ __forceinline__ bool ent_better(long long ka, int ra, long long kb, int rb) {
   return ka > kb || (ka == kb && ra < rb);
 }
@@ -277,36 +296,48 @@ __device__ __noinline__ HeapEnt heap_pop_warp(HeapEnt* h, int n, int lane) {
   return top;
 }
 
-// Min-heap of the K largest latencies seen so far; single lane.  Its root
-// is the K-th largest latency, i.e. the nearest-rank P95 when
-// K = n - ceil(0.95 n) + 1.
-__device__ __noinline__ void topk_insert(int64_t* h, int& n, int kcap, int64_t v) {
-  if (n < kcap) {
-    int i = n++;
-    while (i > 0) {
-      const int par = (i - 1) >> 1;
-      const int64_t pv = h[par];
-      if (pv <= v) break;
-      h[i] = pv;
-      i = par;
-    }
-    h[i] = v;
-  } else if (v > h[0]) {
-    int i = 0;
-    for (;;) {
-      const int l = 2 * i + 1;
-      if (l >= n) break;
-      int ci = l;
-      int64_t cv = h[l];
-      if (l + 1 < n && h[l + 1] < cv) {
-        cv = h[l + 1];
-        ci = l + 1;
+// Min-heap of the K largest latencies seen so far, 32-ary like the local
+// queues; its root is the K-th largest latency, i.e. the nearest-rank P95
+// when K = n - ceil(0.95 n) + 1.  All lanes call with the same v: lane 0
+// writes the heap, every lane writes the same size and root copies.
+__device__ __noinline__ void topk_insert_warp(WarpShared* W, int64_t v, int lane) {
+  int64_t* const h = W->topk;
+  const int n = W->tk;
+  if (n < W->kcap) {
+    // filling: sift up on lane 0 (few levels)
+    if (lane == 0) {
+      int i = n;
+      while (i > 0) {
+        const int par = (i - 1) >> 5;
+        const int64_t pv = h[par];
+        if (pv <= v) break;
+        h[i] = pv;
+        i = par;
       }
-      if (cv >= v) break;
-      h[i] = cv;
-      i = ci;
+      h[i] = v;
     }
-    h[i] = v;
+    __syncwarp();
+    W->tk = n + 1;
+    if (n + 1 == W->kcap) W->tkmin = h[0];
+  } else if (v > W->tkmin) {
+    // v replaces the root and sinks; one lane per child (latencies are >= 0)
+    int i = 0;
+    int64_t root = v;
+    for (;;) {
+      const int first = 32 * i + 1;
+      if (first >= n) break;
+      const int ch = first + lane;
+      const uint64_t cv = ch < n ? (uint64_t)h[ch] : ~0ull;
+      const uint64_t mn = warp_min_u64(cv);
+      if (mn >= (uint64_t)v) break;
+      const int b = __ffs(__ballot_sync(kFull, cv == mn)) - 1;
+      if (i == 0) root = (int64_t)mn;
+      if (lane == 0) h[i] = (int64_t)mn;
+      i = first + b;
+    }
+    if (lane == 0) h[i] = v;
+    __syncwarp();
+    W->tkmin = root;
   }
 }
 
@@ -345,16 +376,16 @@ __device__ __noinline__ int push_pending(WarpShared* W, HeapEnt* arena, int64_t 
   return HX_OK;
 }
 
-// Lane 0: a query's evaluation call finished at `now` (Sec. 4.3's metrics).
-__device__ __noinline__ void finish_query(WarpShared* W, int64_t* topk, int32_t qid, int64_t now, int64_t arrival,
-                                         int64_t deadline) {
-  W->slo_met += now <= deadline ? 1 : 0;
-  W->n_done++;
-  W->makespan = now;
-  W->digest += query_term(qid, now);
-  int tk = W->tk;
-  topk_insert(topk, tk, W->kcap, now - arrival);
-  W->tk = tk;
+// All lanes: a query's evaluation call finished at `now` (Sec. 4.3's metrics).
+__device__ __noinline__ void finish_query(WarpShared* W, int32_t qid, int64_t now, int64_t arrival, int64_t deadline,
+                                         int lane) {
+  if (lane == 0) {
+    W->slo_met += now <= deadline ? 1 : 0;
+    W->n_done++;
+    W->makespan = now;
+  }
+  digest_push(W, now, query_tag(qid), lane);
+  topk_insert_warp(W, now - arrival, lane);
 }
 
 __device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, int m, int64_t now, int64_t budget) {
@@ -459,11 +490,13 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       W->rr = 0;
       W->bump = 0;
       W->digest = 0;
+      W->dn = 0;
       W->makespan = 0;
       W->n_done = 0;
       W->slo_met = 0;
       W->events = 0;
       W->tk = 0;
+      W->tkmin = 0;
     }
     __syncwarp();
 
@@ -542,7 +575,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           rel_first = rid + 1;
           rel_count = k;
         } else if (stg == HX_STAGE_E) {
-          if (lane == 0) finish_query(W, W->topk, qid, now, r->arrival, r->deadline);
+          finish_query(W, qid, now, r->arrival, r->deadline, lane);
         } else {
           const int32_t nx = tail.y;
           if (nx >= 0) {
@@ -701,12 +734,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           if (lane >= pos && lane < cn) sl[lane + 1] = cur;
           if (lane == pos) sl[pos] = nk;
           ++cn;
-          if (lane == 0) {
-            W->digest += call_term(rid, m, now);
-            if (kGeneric) {
-              const int recj = W->recj;
-              if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
-            }
+          digest_push(W, now, call_tag(rid, m), lane);
+          if (kGeneric && lane == 0) {
+            const int recj = W->recj;
+            if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
           }
           __syncwarp();
         }
@@ -716,7 +747,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       if (status != HX_OK) break;
     }
 
-    __syncwarp();
+    digest_flush(W, W->dn, lane);
     if (lane == 0) {
       int st = status;
       const int32_t n_done = W->n_done;
