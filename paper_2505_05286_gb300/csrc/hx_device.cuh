@@ -122,9 +122,9 @@ struct WarpShared {
   int32_t hcap[HX_MAX_INST];    //              heap capacity
   int32_t hsize[HX_MAX_INST];   //              heap size
   int32_t cnt[HX_MAX_INST];     // running calls (the first cnt of the instance's slot keys)
-  // this event's dispatches in order: local-queue key, (request id, service time)
-  int64_t pkey[32];
+  // this event's dispatches in order: (request id, service time), Eq. (comp) on the winner
   int2 prs[32];
+  int32_t pest[32];
   // per-simulation constants
   int64_t A, one_minus_a, G, beta;
   int64_t frest[kFRows];        // rest-of-path cost of the budget denominator by fcode

@@ -344,12 +344,41 @@ __device__ __noinline__ void topk_insert_warp(WarpShared* W, int64_t v, int lane
 // Queue this event's dispatches to instance m (pending entries on the lanes of
 // mask pm) in m's heap, re-homing the heap in the arena when it is full.
 // All lanes call.  Returns HX_OK or HX_ERR_CAPACITY.
-__device__ __noinline__ int push_pending(WarpShared* W, HeapEnt* arena, int64_t arena_per_warp, int m, unsigned pm,
-                                        int lane) {
+__device__ __noinline__ int64_t budget_wide(int64_t num, int64_t tb, int64_t d) { return scaled_div(num, tb, d); }
+
+// t_slo of Eq. (budget): (deadline - now) * tbar / (tbar + F), truncated
+// toward zero; |num| < 2^34 keeps |num| * tbar below 2^63.
+__device__ __forceinline__ int64_t slo_budget(int64_t num, int64_t tb, int64_t dd) {
+  if (num > -(int64_t(1) << 34) && num < (int64_t(1) << 34)) {
+    const uint64_t res = udiv_trial((uint64_t)(num < 0 ? -num : num) * (uint64_t)tb, (uint64_t)dd);
+    return num < 0 ? -(int64_t)res : (int64_t)res;
+  }
+  return budget_wide(num, tb, dd);
+}
+
+// The instance's new requests (pending entries, bits of pm) join its local
+// queue.  Their keys, higher first, are formed here, one per lane: Eq.
+// (priority) with the budget at send time (now) and the common now dropped;
+// FCFS: earliest enqueue; LLF: least deadline - now - remaining work, again
+// with the common now dropped.
+__device__ __noinline__ int push_pending(WarpShared* W, const CallRec* rec, int64_t now, int lpol,
+                                        int64_t arena_per_warp, int m, unsigned pm, int lane) {
+  long long key = 0;
+  if ((pm >> lane) & 1u) {
+    const CallRec* r = rec + W->prs[lane].x;
+    const int64_t dl = r->deadline;
+    const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
+    const int64_t tb = tail.x;
+    const int64_t dd = tb + W->frest[(uint32_t)tail.w >> 24];
+    key = lpol == HX_LOCAL_PQ     ? (long long)(kScale * ((int64_t)W->pest[lane] - slo_budget(dl - now, tb, dd)) - W->G * now)
+          : lpol == HX_LOCAL_FCFS ? (long long)(-now)
+                                  : (long long)(dd - dl);
+  }
+  HeapEnt* const arena = W->arena;
   while (pm) {
     const int j = __ffs(pm) - 1;
     pm &= pm - 1;
-    const long long key = W->pkey[j];
+    const long long kj = __shfl_sync(kFull, key, j);
     const int2 rs = W->prs[j];
     const int rid = rs.x, svc = rs.y;
     const int size = W->hsize[m], cap = W->hcap[m], off = W->hoff[m], bump = W->bump;
@@ -368,7 +397,7 @@ __device__ __noinline__ int push_pending(WarpShared* W, HeapEnt* arena, int64_t 
       }
     }
     if (lane == 0) {
-      heap_push(arena + hoff, size, key, rid, svc);
+      heap_push(arena + hoff, size, kj, rid, svc);
       W->hsize[m] = size + 1;
     }
     __syncwarp();
@@ -395,7 +424,6 @@ __device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, i
   a.rec_budget[o] = budget;
 }
 
-__device__ __noinline__ int64_t budget_wide(int64_t num, int64_t tb, int64_t d) { return scaled_div(num, tb, d); }
 
 }  // namespace
 
@@ -603,51 +631,32 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         W->akey = qa + 1 < W->nq ? (((uint64_t)a.arrival[qbase + qa + 1] << 7) | kArrivalTag) : kKeyInf;
       }
 
-      // Sec. 4.1 + 4.2 for each released request, in request-id order: budget at
-      // send time, score every instance, enqueue on the winner.
+      // Sec. 4.1 for each released request, in request-id order: score every
+      // instance and send it to the winner (its Sec. 4.2 key is formed at the
+      // batch boundary below, and only if it has to wait).
       for (int32_t jr = 0; jr < rel_count; ++jr) {
         const int32_t rid = rel_first + jr;
         const CallRec* r = rec + rid;
         // Eq. (comp) and the service time on this lane's two instances
         const int e0 = r->est[ty0], e1 = r->est[ty1];
         const int v0 = r->svc[ty0], v1 = r->svc[ty1];
-        const int64_t dl = r->deadline;
-        const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
-        const int64_t tb = tail.x;
-        const int64_t dd = tb + W->frest[(uint32_t)tail.w >> 24];
-        const int64_t num = dl - now;
-        const bool small = num > -(int64_t(1) << 34) && num < (int64_t(1) << 34);
-        // SIMT division passes: each lane refreshes one stale reward of its
-        // instances per pass; the budget goes to the lowest lane with nothing
-        // stale.  Two passes at most clear the rewards, three the budget.
-        int64_t bres = 0;
-        bool need_budget = small;
-        int bl = 0;
-        const uint64_t beta = (uint64_t)W->beta;
         if (W->one_minus_a == 0 || (kGeneric && W->dpol == HX_DISPATCH_RR)) {
           // rewards carry no weight at alpha = 1 and are unused by round robin
           dirty0 = false;
           dirty1 = false;
         }
-        const uint64_t bn = (uint64_t)(num < 0 ? -num : num) * (uint64_t)tb;
-        for (;;) {
+        // SIMT division passes: each lane refreshes one stale reward of its
+        // instances per pass (two passes at most)
+        const uint64_t beta = (uint64_t)W->beta;
+        while (__any_sync(kFull, dirty0 || dirty1)) {
           const bool rj = dirty0 || dirty1;
-          const unsigned busy = __ballot_sync(kFull, rj);
-          const int cand = (need_budget && ~busy) ? __ffs(~busy) - 1 : -1;
-          const bool bj = lane == cand;  // never a lane with a stale reward
           const int64_t q = W->q[dirty0 ? m0 : m1];
-          const uint64_t n = rj ? beta : (bj ? bn : 0);
-          const uint64_t d = rj ? (uint64_t)(q > 1 ? q : 1) : (bj ? (uint64_t)dd : 1);
-          const uint64_t res = udiv_trial(n, d);
+          const uint64_t res = udiv_trial(rj ? beta : 0ull, (rj && q > 1) ? (uint64_t)q : 1ull);
           const int64_t orew =
               (int64_t)(int32_t)W->one_minus_a * (res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap);
           if (dirty0) { orew0 = orew; dirty0 = false; }
           else if (dirty1) { orew1 = orew; dirty1 = false; }
-          if (bj) bres = num < 0 ? -(int64_t)res : (int64_t)res;
-          if (cand >= 0) { bl = cand; need_budget = false; }
-          if (!need_budget && !__any_sync(kFull, dirty0 || dirty1)) break;
         }
-        const int64_t budget = small ? __shfl_sync(kFull, bres, bl) : budget_wide(num, tb, dd);
         int m;
         if (kGeneric && W->dpol == HX_DISPATCH_RR) {
           m = W->rr;
@@ -668,25 +677,23 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           if (m < 32) dirty0 = true;
           else dirty1 = true;
         }
-        // local-queue key, higher first: Eq. (priority) aged by gamma with the
-        // common now dropped; FCFS: earliest enqueue; LLF: least deadline - now -
-        // remaining work, again with the common now dropped
-        const int lpol = kGeneric ? W->lpol : HX_LOCAL_PQ;
-        const long long key = lpol == HX_LOCAL_PQ     ? (long long)(kScale * (est_m - budget) - W->G * now)
-                              : lpol == HX_LOCAL_FCFS ? (long long)(-now)
-                                                      : (long long)(dd - dl);
+        // the local-queue key is formed only if the request has to wait
         if (lane == npend) {
           pend_m = m;
         }
         if (lane == 0) {
-          W->pkey[npend] = key;
           W->prs[npend] = make_int2(rid, svc_m);
+          W->pest[npend] = (int32_t)est_m;
         }
         npend++;
         touched |= 1ull << m;
         if (kGeneric) {
           const int recj = W->recj;
-          if (recj >= 0 && lane == 0) log_dispatch(a, recj, rid, m, now, budget);
+          if (recj >= 0) {
+            const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
+            const int64_t budget = slo_budget(r->deadline - now, tail.x, tail.x + W->frest[(uint32_t)tail.w >> 24]);
+            if (lane == 0) log_dispatch(a, recj, rid, m, now, budget);
+          }
         }
       }
 
@@ -705,7 +712,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         // fast path: an empty queue with room for all of this event's arrivals
         const bool direct = hs == 0 && __popc(pm) <= ns - cn;
         if (!direct && pm) {
-          status = push_pending(W, W->arena, a.arena_per_warp, m, pm, lane);
+          status = push_pending(W, rec, now, kGeneric ? W->lpol : HX_LOCAL_PQ, a.arena_per_warp, m, pm, lane);
           if (status != HX_OK) break;
         }
         unsigned bits = direct ? pm : 0u;
