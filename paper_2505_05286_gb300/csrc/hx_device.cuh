@@ -22,6 +22,8 @@ constexpr int64_t kScale = 1000000;       // fixed point of alpha, gamma, slo_mu
 constexpr int64_t kUsPerS = 1000000;      // prefill throughput is per second
 constexpr int64_t kRewardCap = (int64_t(1) << 43) - 1;
 constexpr uint64_t kKeyInf = ~0ull;
+// Event keys (time << 7 | instance) stay below 2^46: every time is below 2^39.
+constexpr uint64_t kNoEvent = 1ull << 46;
 constexpr int64_t kTimeInf = INT64_MAX;
 constexpr int kWarpsPerBlock = 4;
 constexpr unsigned kFull = 0xffffffffu;

@@ -49,11 +49,12 @@ __device__ __forceinline__ int warp_argmax_s64(int64_t s, int idx) {
 
 // floor(n / d) for 0 <= n < 2^63 and 1 <= d < 2^54.  Trial-quotient method
 // (Knuth, TAOCP vol. 2, 4.3.1): a quotient estimate from a single-precision
-// reciprocal, refined once on the exact int64 remainder, then corrected by at
-// most one step each way.  Operands reach float through two 32-bit halves.
-// Estimate error: |q0 - n/d| < 2^30 * 2^-21 + 1, so the remainder fits int64
-// and the refined quotient is within one of n/d.  Quotients of 2^30 or more
-// (and d = 1) take the exact integer paths.
+// reciprocal, refined once on the exact int64 remainder when it is 2^21 or
+// more, then corrected by at most one step each way.  Operands reach float
+// through two 32-bit halves.  The estimate's relative error is below
+// 3.5 * 2^-23 (two conversions, the approximate reciprocal, one product), so
+// below 2^21 it is within one of n/d, and below 2^30 the refined one is.
+// Quotients of 2^30 or more (and d = 1) take the exact integer paths.
 __device__ __forceinline__ float u64_to_float(uint64_t x) {
   return __fmaf_rn((float)(uint32_t)(x >> 32), 4294967296.0f, (float)(uint32_t)x);
 }
@@ -70,8 +71,10 @@ __device__ __forceinline__ uint64_t udiv_trial(uint64_t n, uint64_t d) {
   if (qf >= 1073741824.0f) return n / d;
   uint64_t q = (uint32_t)qf;
   int64_t r = (int64_t)(n - q * d);
-  q += (int64_t)(int32_t)(s64_to_float(r) * rd);
-  r = (int64_t)(n - q * d);
+  if (qf >= 2097152.0f) {
+    q += (int64_t)(int32_t)(s64_to_float(r) * rd);
+    r = (int64_t)(n - q * d);
+  }
   if (r < 0) {
     q--;
     r += (int64_t)d;
@@ -552,7 +555,8 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
 
     auto set_key = [&](int m, uint64_t nk) {
       if (lane == (m & 31)) {
-        const uint64_t kk = nk == kKeyInf ? kKeyInf : (((nk >> 24) << 7) | (uint64_t)m);
+        // an empty instance (nk all ones) maps to a key at or above kNoEvent
+        const uint64_t kk = ((nk >> 24) << 7) | (uint64_t)m;
         if (m < 32) k0 = kk; else k1 = kk;
       }
     };
@@ -560,7 +564,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     for (;;) {
       const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
       const uint64_t akey = W->akey;
-      if (ck == kKeyInf && akey == kKeyInf) break;
+      if (ck >= kNoEvent && akey == kKeyInf) break;
       if (--steps_left < 0) {
         status = HX_ERR_STEP_LIMIT;
         break;

@@ -22,6 +22,11 @@ def _cases(rng, count):
     n[2 * k:3 * k] = (n[2 * k:3 * k] % np.uint64(2 ** 40)) // d[2 * k:3 * k] * d[2 * k:3 * k] + d[2 * k:3 * k] - np.uint64(1)
     d[3 * k:4 * k] = 1
     d[4 * k:5 * k] = rng.integers(1, 1000, k, dtype=np.uint64)
+    # quotients near the 2^21 switch (one refinement step below it), small and
+    # large divisors, any remainder
+    d2 = (rng.integers(1, 2 ** 40, k, dtype=np.uint64) >> rng.integers(0, 40, k).astype(np.uint64)) + np.uint64(1)
+    q2 = (np.uint64(2 ** 21) + rng.integers(-4, 4, k).astype(np.int64).astype(np.uint64))
+    n[5 * k:6 * k], d[5 * k:6 * k] = d2 * q2 + rng.integers(0, 2 ** 62, k, dtype=np.uint64) % d2, d2
     return n, d
 
 
