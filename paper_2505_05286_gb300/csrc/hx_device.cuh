@@ -121,12 +121,12 @@ struct SimArgs {
 struct WarpShared {
   int64_t q[HX_MAX_INST];       // t_queue: Eq. comp summed over requests dispatched and unfinished
   int32_t hoff[HX_MAX_INST];    // local queue: heap offset in the arena
-  int32_t hcap[HX_MAX_INST];    //              heap capacity
   int32_t hsize[HX_MAX_INST];   //              heap size
-  int32_t cnt[HX_MAX_INST];     // running calls (the first cnt of the instance's slot keys)
+  uint8_t cnt[HX_MAX_INST];     // running calls (the first cnt of the instance's slot keys)
+  uint8_t hcl[HX_MAX_INST];     // local queue: heap capacity 8 << hcl (0: none yet)
   // this event's dispatches in order: (request id, service time), Eq. (comp) on the winner
-  int2 prs[32];
-  int32_t pest[32];
+  int2 prs[HX_MAX_K];
+  int32_t pest[HX_MAX_K];
   // per-simulation constants
   int64_t A, one_minus_a, G, beta;
   int64_t frest[kFRows];        // rest-of-path cost of the budget denominator by fcode
@@ -145,8 +145,8 @@ struct WarpShared {
   int64_t makespan;
   int32_t n_done, slo_met, events, tk;
   int64_t tkmin;                // root of the full top-K heap (written alike by every lane)
-  int64_t dt[32];               // digest terms waiting to be hashed: time, id tag
-  uint32_t dtag[32];
+  int64_t dt[16];               // digest terms waiting to be hashed: time, id tag
+  uint32_t dtag[16];
   int32_t dn, pad1;             // terms waiting (written alike by every lane)
   uint64_t slot[1];             // [total_slots]
 };

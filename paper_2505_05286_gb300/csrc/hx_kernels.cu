@@ -207,7 +207,7 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
 // -------------------------------------------------------- simulation kernel
 namespace {
 
-// The digest is a sum of terms, so they are hashed 32 at a time: every lane
+// The digest is a sum of terms, so they are hashed 16 at a time: every lane
 // calls with the same (t, tag); lane 0 appends it, and a full batch is hashed
 // one term per lane and summed into W->digest.
 __device__ __noinline__ void digest_flush(WarpShared* W, int n, int lane) {
@@ -226,7 +226,7 @@ __device__ __forceinline__ void digest_push(WarpShared* W, int64_t t, uint32_t t
     W->dt[n] = t;
     W->dtag[n] = tag;
   }
-  if (n == 31) digest_flush(W, 32, lane);
+  if (n == 15) digest_flush(W, 16, lane);
   else W->dn = n + 1;
 }
 
@@ -238,7 +238,7 @@ __device__ __forceinline__ bool ent_better(long long ka, int ra, long long kb, i
 // arena: node i has children 32 i + 1 .. 32 i + 32, so 40k waiting requests
 // sit four levels deep.  Push sifts up on one lane (new requests rarely
 // climb); pop sifts down with the whole warp, one lane per child.
-__device__ __noinline__ void heap_push(HeapEnt* h, int n, long long key, int rid, int svc) {
+__device__ __forceinline__ void heap_push(HeapEnt* h, int n, long long key, int rid, int svc) {
   int i = n;
   while (i > 0) {
     const int par = (i - 1) >> 5;
@@ -384,7 +384,8 @@ __device__ __noinline__ int push_pending(WarpShared* W, const CallRec* rec, int6
     const long long kj = __shfl_sync(kFull, key, j);
     const int2 rs = W->prs[j];
     const int rid = rs.x, svc = rs.y;
-    const int size = W->hsize[m], cap = W->hcap[m], off = W->hoff[m], bump = W->bump;
+    const int size = W->hsize[m], hcl = W->hcl[m], off = W->hoff[m], bump = W->bump;
+    const int cap = hcl ? 8 << hcl : 0;
     __syncwarp();
     int hoff = off;
     if (size == cap) {
@@ -396,7 +397,7 @@ __device__ __noinline__ int push_pending(WarpShared* W, const CallRec* rec, int6
       if (lane == 0) {
         W->bump = bump + ncap;
         W->hoff[m] = hoff;
-        W->hcap[m] = ncap;
+        W->hcl[m] = (uint8_t)(hcl + 1);
       }
     }
     if (lane == 0) {
@@ -480,7 +481,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
 
     for (int m = lane; m < 64; m += 32) {
       W->hoff[m] = 0;
-      W->hcap[m] = 0;
+      W->hcl[m] = 0;
       W->hsize[m] = 0;
       W->cnt[m] = 0;
     }
