@@ -270,7 +270,7 @@ def run_gpu(args):
     roofline = {"bound": "alu", "achieved": achieved / 1e9, "peak": peak / 1e9, "unit": "Gwarp-inst/s",
                 "frac": achieved / peak, "traffic": _traffic_per_launch(wl.n_sims),
                 "work_per_event": WARP_INST_PER_EVENT, "events_per_launch": events_per_step,
-                "kernel": "hx_sim_kernel", "kernel_ms": kern_ms,
+                "kernel": "hx_sim_kernel" if info["generic_kernel"] else "hx_sim_kernel_lean", "kernel_ms": kern_ms,
                 "peak_source": f"{sm_count} SMs x 4 schedulers x {sm_mhz:.0f} MHz ({peak_kind} sm_max_mhz)"}
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",

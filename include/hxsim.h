@@ -255,6 +255,9 @@ typedef struct hx_info {
   int32_t warps_per_block;
   int32_t blocks;
   int32_t smem_per_block;
+  int32_t generic_kernel;       /* 1: the kernel with logging and every policy; 0: the
+                                   PQ + workload-balanced instantiation without logging */
+  int32_t reserved;
 } hx_info;
 
 int hx_sim_info(hx_sim* h, hx_info* out);

@@ -715,6 +715,8 @@ int hx_sim_info(hx_sim* h, hx_info* out) {
   out->warps_per_block = hx::kWarpsPerBlock;
   out->blocks = h->blocks;
   out->smem_per_block = h->smem_per_block;
+  out->generic_kernel = h->generic ? 1 : 0;
+  out->reserved = 0;
   return HX_OK;
 }
 

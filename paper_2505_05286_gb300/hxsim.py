@@ -73,7 +73,8 @@ class hx_info(ctypes.Structure):
                 ("n_queries_total", ctypes.c_int64), ("scratch_bytes", ctypes.c_int64),
                 ("device_bytes", ctypes.c_int64), ("resident_warps", ctypes.c_int32),
                 ("warps_per_block", ctypes.c_int32), ("blocks", ctypes.c_int32),
-                ("smem_per_block", ctypes.c_int32)]
+                ("smem_per_block", ctypes.c_int32), ("generic_kernel", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
 
 
 _lib = None

@@ -42,7 +42,7 @@ int main(void) {
   S(hx_options) F(hx_options, record_sims) F(hx_options, timing) F(hx_options, force_generic)
   S(hx_result) F(hx_result, digest) F(hx_result, status) F(hx_result, cycles_k)
   S(hx_best) F(hx_best, global_sum_p95) F(hx_best, per_trace_point)
-  S(hx_info) F(hx_info, resident_warps) F(hx_info, smem_per_block)
+  S(hx_info) F(hx_info, resident_warps) F(hx_info, smem_per_block) F(hx_info, generic_kernel)
   return 0;
 }
 """
