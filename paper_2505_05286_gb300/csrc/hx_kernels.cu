@@ -236,7 +236,7 @@ __device__ __forceinline__ bool ent_better(long long ka, int ra, long long kb, i
 
 // Local queues are 32-ary max-heaps on (key desc, rid asc) in the warp's
 // arena: node i has children 32 i + 1 .. 32 i + 32, so 40k waiting requests
-// sit four levels deep.  Push sifts up on one lane (new requests rarely
+// climb); pop and replace sift down with the whole warp, one lane per child.
 // climb); pop sifts down with the whole warp, one lane per child.
 __device__ __forceinline__ void heap_push(HeapEnt* h, int n, long long key, int rid, int svc) {
   int i = n;
@@ -254,11 +254,12 @@ __device__ __forceinline__ void heap_push(HeapEnt* h, int n, long long key, int 
   h[i] = e;
 }
 
-// All lanes call with the same (h, n >= 1); every lane gets the top entry.
-__device__ __noinline__ HeapEnt heap_pop_warp(HeapEnt* h, int n, int lane) {
+// All lanes call with the same arguments.  The top entry leaves the heap and
+// `sink` takes its place, sinking to its level; the heap then holds m
+// entries (m = n - 1 and sink = the last entry: a pop; m = n and sink = a new
+// entry: a replace).  Every lane gets the old top.
+__device__ __noinline__ HeapEnt heap_sift_warp(HeapEnt* h, int m, HeapEnt sink, int lane) {
   const HeapEnt top = h[0];
-  const HeapEnt last = h[n - 1];
-  const int m = n - 1;
   int i = 0;
   for (;;) {
     const int first = 32 * i + 1;
@@ -272,29 +273,31 @@ __device__ __noinline__ HeapEnt heap_pop_warp(HeapEnt* h, int n, int lane) {
       cr = e.rid;
       cs = e.svc;
     }
-    // warp argmax of (key desc, rid asc)
+    // warp argmax of (key desc, rid asc): the rids decide only among equal keys
     const uint64_t uk = (uint64_t)ck ^ 0x8000000000000000ull;
     const uint32_t hi = (uint32_t)(uk >> 32), lo = (uint32_t)uk;
     const uint32_t mh = __reduce_max_sync(kFull, hi);
     const bool c1 = hi == mh;
     const uint32_t ml = __reduce_max_sync(kFull, c1 ? lo : 0u);
-    const bool c2 = c1 && lo == ml;
-    const uint32_t mr = __reduce_min_sync(kFull, c2 ? (uint32_t)cr : 0xffffffffu);
-    const int b = __ffs(__ballot_sync(kFull, c2 && (uint32_t)cr == mr)) - 1;
-    const long long bk = __shfl_sync(kFull, ck, b);
-    const int br = __shfl_sync(kFull, cr, b);
-    const int bs = __shfl_sync(kFull, cs, b);
-    if (!ent_better(bk, br, last.key, last.rid)) break;
-    if (lane == 0) {
+    unsigned best = __ballot_sync(kFull, c1 && lo == ml);
+    if (best & (best - 1)) {
+      const bool tie = (best >> lane) & 1u;
+      const uint32_t mr = __reduce_min_sync(kFull, tie ? (uint32_t)cr : 0xffffffffu);
+      best = __ballot_sync(kFull, tie && (uint32_t)cr == mr);
+    }
+    const int b = __ffs(best) - 1;
+    // the best child moves up unless the sinking entry goes before it
+    if (!__shfl_sync(kFull, (int)ent_better(ck, cr, sink.key, sink.rid), b)) break;
+    if (lane == b) {
       HeapEnt e;
-      e.key = bk;
-      e.rid = br;
-      e.svc = bs;
+      e.key = ck;
+      e.rid = cr;
+      e.svc = cs;
       h[i] = e;
     }
     i = first + b;
   }
-  if (lane == 0 && m > 0) h[i] = last;
+  if (lane == 0 && m > 0) h[i] = sink;
   __syncwarp();
   return top;
 }
@@ -359,24 +362,27 @@ __device__ __forceinline__ int64_t slo_budget(int64_t num, int64_t tb, int64_t d
   return budget_wide(num, tb, dd);
 }
 
+// Local-queue key, higher first, of pending entry j: Eq. (priority) with
+// the budget at send time (now) and the common now dropped; FCFS: earliest
+// enqueue; LLF: least deadline - now - remaining work, again with the common
+// now dropped.
+__device__ __forceinline__ long long pending_key(const WarpShared* W, const CallRec* rec, int64_t now, int lpol,
+                                                 int j) {
+  const CallRec* r = rec + W->prs[j].x;
+  const int64_t dl = r->deadline;
+  const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
+  const int64_t tb = tail.x;
+  const int64_t dd = tb + W->frest[(uint32_t)tail.w >> 24];
+  return lpol == HX_LOCAL_PQ     ? (long long)(kScale * ((int64_t)W->pest[j] - slo_budget(dl - now, tb, dd)) - W->G * now)
+         : lpol == HX_LOCAL_FCFS ? (long long)(-now)
+                                 : (long long)(dd - dl);
+}
+
 // The instance's new requests (pending entries, bits of pm) join its local
-// queue.  Their keys, higher first, are formed here, one per lane: Eq.
-// (priority) with the budget at send time (now) and the common now dropped;
-// FCFS: earliest enqueue; LLF: least deadline - now - remaining work, again
-// with the common now dropped.
+// queue, their keys formed one per lane.
 __device__ __noinline__ int push_pending(WarpShared* W, const CallRec* rec, int64_t now, int lpol,
                                         int64_t arena_per_warp, int m, unsigned pm, int lane) {
-  long long key = 0;
-  if ((pm >> lane) & 1u) {
-    const CallRec* r = rec + W->prs[lane].x;
-    const int64_t dl = r->deadline;
-    const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
-    const int64_t tb = tail.x;
-    const int64_t dd = tb + W->frest[(uint32_t)tail.w >> 24];
-    key = lpol == HX_LOCAL_PQ     ? (long long)(kScale * ((int64_t)W->pest[lane] - slo_budget(dl - now, tb, dd)) - W->G * now)
-          : lpol == HX_LOCAL_FCFS ? (long long)(-now)
-                                  : (long long)(dd - dl);
-  }
+  const long long key = ((pm >> lane) & 1u) ? pending_key(W, rec, now, lpol, lane) : 0;
   HeapEnt* const arena = W->arena;
   while (pm) {
     const int j = __ffs(pm) - 1;
@@ -407,6 +413,26 @@ __device__ __noinline__ int push_pending(WarpShared* W, const CallRec* rec, int6
     __syncwarp();
   }
   return HX_OK;
+}
+
+// One new request (the single bit of pm) meets an instance with one free slot
+// and a non-empty local queue: the more urgent of it and the queue's top
+// starts and the other waits, i.e. a push and a pop in one sift (the new
+// request replaces the top).  Returns the started (request id, service time).
+__device__ __noinline__ int2 push_pop(WarpShared* W, const CallRec* rec, int64_t now, int lpol, int m, unsigned pm,
+                                     int lane) {
+  const int j = __ffs(pm) - 1;
+  const long long key = __shfl_sync(kFull, lane == j ? pending_key(W, rec, now, lpol, j) : 0, j);
+  const int2 rs = W->prs[j];
+  HeapEnt* const h = W->arena + W->hoff[m];
+  const HeapEnt top = h[0];
+  if (ent_better(key, rs.x, top.key, top.rid)) return rs;
+  HeapEnt e;
+  e.key = key;
+  e.rid = rs.x;
+  e.svc = rs.y;
+  heap_sift_warp(h, W->hsize[m], e, lane);
+  return make_int2(top.rid, top.svc);
 }
 
 // All lanes: a query's evaluation call finished at `now` (Sec. 4.3's metrics).
@@ -714,27 +740,35 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         __syncwarp();
         int cn = W->cnt[m];
         const int hs = W->hsize[m];
-        // fast path: an empty queue with room for all of this event's arrivals
-        const bool direct = hs == 0 && __popc(pm) <= ns - cn;
-        if (!direct && pm) {
-          status = push_pending(W, rec, now, kGeneric ? W->lpol : HX_LOCAL_PQ, a.arena_per_warp, m, pm, lane);
+        // fast paths: an empty queue with room for all of this event's arrivals;
+        // one arrival, one free slot and a waiting queue (one sift)
+        const int npm = __popc(pm);
+        const bool direct = hs == 0 && npm <= ns - cn;
+        const bool fused = !direct && npm == 1 && ns - cn == 1;
+        const int lpol = kGeneric ? W->lpol : HX_LOCAL_PQ;
+        unsigned bits = direct ? pm : 0u;
+        int2 fst = make_int2(0, 0);
+        if (fused) {
+          fst = push_pop(W, rec, now, lpol, m, pm, lane);
+          bits = 1u;
+        } else if (!direct && pm) {
+          status = push_pending(W, rec, now, lpol, a.arena_per_warp, m, pm, lane);
           if (status != HX_OK) break;
         }
-        unsigned bits = direct ? pm : 0u;
         for (;;) {
           int rid, svc;
-          if (direct) {
+          if (direct || fused) {
             if (!bits) break;
             const int j = __ffs(bits) - 1;
             bits &= bits - 1;
-            const int2 rs = W->prs[j];
+            const int2 rs = fused ? fst : W->prs[j];
             rid = rs.x;
             svc = rs.y;
           } else {
             const int n = W->hsize[m];
             __syncwarp();
             if (cn >= ns || n == 0) break;
-            const HeapEnt top = heap_pop_warp(W->arena + W->hoff[m], n, lane);
+            const HeapEnt top = heap_sift_warp(W->arena + W->hoff[m], n - 1, W->arena[W->hoff[m] + n - 1], lane);
             if (lane == 0) W->hsize[m] = n - 1;
             rid = top.rid;
             svc = top.svc;
