@@ -236,8 +236,8 @@ __device__ __forceinline__ bool ent_better(long long ka, int ra, long long kb, i
 
 // Local queues are 32-ary max-heaps on (key desc, rid asc) in the warp's
 // arena: node i has children 32 i + 1 .. 32 i + 32, so 40k waiting requests
+// sit four levels deep.  Push sifts up on one lane (new requests rarely
 // climb); pop and replace sift down with the whole warp, one lane per child.
-// climb); pop sifts down with the whole warp, one lane per child.
 __device__ __forceinline__ void heap_push(HeapEnt* h, int n, long long key, int rid, int svc) {
   int i = n;
   while (i > 0) {
