@@ -128,7 +128,9 @@ struct WarpShared {
   int2 prs[HX_MAX_K];
   int32_t pest[HX_MAX_K];
   // per-simulation constants
-  int64_t A, one_minus_a, G, beta;
+  int32_t A, one_minus_a;        // alpha and 1 - alpha, fixed point
+  int32_t rewards, pad2;          // 1 when dispatch scores need the reward term
+  int64_t G, beta;
   int64_t frest[kFRows];        // rest-of-path cost of the budget denominator by fcode
   int32_t lpol, dpol, recj, kcap, rr, bump;
   // this warp's scratch slices and the current trace's offsets
@@ -145,8 +147,7 @@ struct WarpShared {
   int64_t makespan;
   int32_t n_done, slo_met, events, tk;
   int64_t tkmin;                // root of the full top-K heap (written alike by every lane)
-  int64_t dt[16];               // digest terms waiting to be hashed: time, id tag
-  uint32_t dtag[16];
+  longlong2 dterm[16];          // digest terms waiting to be hashed: (time, id tag)
   int32_t dn, pad1;             // terms waiting (written alike by every lane)
   uint64_t slot[1];             // [total_slots]
 };

@@ -212,7 +212,8 @@ namespace {
 // one term per lane and summed into W->digest.
 __device__ __noinline__ void digest_flush(WarpShared* W, int n, int lane) {
   __syncwarp();
-  uint64_t y = lane < n ? digest_term((uint64_t)W->dt[lane], W->dtag[lane]) : 0ull;
+  const longlong2 e = W->dterm[lane < n ? lane : 0];
+  uint64_t y = lane < n ? digest_term((uint64_t)e.x, (uint64_t)e.y) : 0ull;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) y += __shfl_xor_sync(kFull, y, o);
   if (lane == 0) W->digest += y;
@@ -222,10 +223,7 @@ __device__ __noinline__ void digest_flush(WarpShared* W, int n, int lane) {
 
 __device__ __forceinline__ void digest_push(WarpShared* W, int64_t t, uint32_t tag, int lane) {
   const int n = W->dn;
-  if (lane == 0) {
-    W->dt[n] = t;
-    W->dtag[n] = tag;
-  }
+  if (lane == 0) W->dterm[n] = make_longlong2(t, (long long)tag);
   if (n == 15) digest_flush(W, 16, lane);
   else W->dn = n + 1;
 }
@@ -537,8 +535,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     }
     if (lane == 0) {
       const int64_t A = a.alpha[p];
-      W->A = A;
-      W->one_minus_a = kScale - A;
+      W->A = (int32_t)A;
+      W->one_minus_a = (int32_t)(kScale - A);
+      // rewards carry no weight at alpha = 1 and are unused by round robin
+      W->rewards = (A != kScale && !(kGeneric && a.dpol[p] == HX_DISPATCH_RR)) ? 1 : 0;
       W->G = a.gamma[p];
       W->beta = a.beta[p];
       W->lpol = a.lpol[p];
@@ -564,7 +564,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     W->q[m1] = 0;
     // (1 - alpha) * reward per instance; instances past N score far below any
     // real one (|alpha * est| < 2^52), so the argmax needs no validity test
-    const int32_t oma32 = (int32_t)W->one_minus_a;
+    const int32_t oma32 = W->one_minus_a;
     const int64_t orew_idle = (int64_t)oma32 * reward_of(W->beta, 0);
     int64_t orew0 = valid0 ? orew_idle : -(int64_t(1) << 62);
     int64_t orew1 = valid1 ? orew_idle : -(int64_t(1) << 62);
@@ -615,14 +615,16 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         const int hs_m = W->hsize[m];
         // remove it: the remaining keys move down one slot
         const uint64_t nxt = lane + 1 < cn ? sl[lane + 1] : kKeyInf;
+        const uint64_t head = cn > 1 ? sl[1] : kKeyInf;
         __syncwarp();
         if (lane < cn) sl[lane] = nxt;
         if (lane == 0) W->cnt[m] = cn - 1;
-        set_key(m, __shfl_sync(kFull, nxt, 0));
+        set_key(m, head);
         if (lane == (m & 31)) {
           W->q[m] -= est_m;
-          if (m < 32) dirty0 = true;
-          else dirty1 = true;
+          const bool stale = W->rewards != 0;
+          if (m < 32) dirty0 = stale;
+          else dirty1 = stale;
         }
         // the freed slot needs a batch boundary only if requests wait for it
         if (hs_m > 0) touched |= 1ull << m;
@@ -641,13 +643,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             rel_first = nx;
             rel_count = 1;
           } else {
-            int left = 0;
-            if (lane == 0) {
-              uint8_t* const chains = W->chains;
-              left = chains[qid] - 1;
-              chains[qid] = (uint8_t)left;
-            }
-            left = __shfl_sync(kFull, left, 0);
+            uint8_t* const chains = W->chains;
+            const int left = chains[qid] - 1;
+            __syncwarp();
+            if (lane == 0) chains[qid] = (uint8_t)left;
             rel_first = ~nx;
             rel_count = left == 0 ? 1 : 0;
           }
@@ -671,11 +670,6 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         // Eq. (comp) and the service time on this lane's two instances
         const int e0 = r->est[ty0], e1 = r->est[ty1];
         const int v0 = r->svc[ty0], v1 = r->svc[ty1];
-        if (W->one_minus_a == 0 || (kGeneric && W->dpol == HX_DISPATCH_RR)) {
-          // rewards carry no weight at alpha = 1 and are unused by round robin
-          dirty0 = false;
-          dirty1 = false;
-        }
         // SIMT division passes: each lane refreshes one stale reward of its
         // instances per pass (two passes at most)
         const uint64_t beta = (uint64_t)W->beta;
@@ -684,7 +678,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           const int64_t q = W->q[dirty0 ? m0 : m1];
           const uint64_t res = udiv_trial(rj ? beta : 0ull, (rj && q > 1) ? (uint64_t)q : 1ull);
           const int64_t orew =
-              (int64_t)(int32_t)W->one_minus_a * (res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap);
+              (int64_t)W->one_minus_a * (res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap);
           if (dirty0) { orew0 = orew; dirty0 = false; }
           else if (dirty1) { orew1 = orew; dirty1 = false; }
         }
@@ -694,7 +688,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           __syncwarp();
           if (lane == 0) W->rr = (m + 1 == N) ? 0 : m + 1;
         } else {
-          const int32_t A = (int32_t)W->A;
+          const int32_t A = W->A;
           const int64_t s0 = orew0 - (int64_t)A * e0;
           const int64_t s1 = orew1 - (int64_t)A * e1;
           const bool take1 = s1 > s0;
@@ -705,8 +699,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         const int svc_m = __shfl_sync(kFull, m < 32 ? v0 : v1, m & 31);
         if (lane == (m & 31)) {
           W->q[m] += est_m;
-          if (m < 32) dirty0 = true;
-          else dirty1 = true;
+          const bool stale = W->rewards != 0;
+          if (m < 32) dirty0 = stale;
+          else dirty1 = stale;
         }
         // the local-queue key is formed only if the request has to wait
         if (lane == npend) {
