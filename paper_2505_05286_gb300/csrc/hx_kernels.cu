@@ -580,6 +580,22 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     uint64_t touched = 0;
     int32_t steps_left = nc + nq + 8;
 
+    // Request rid starts on instance m now and runs until now + svc: its key
+    // joins the cn sorted keys of m's running calls at sl.
+    auto start_call = [&](uint64_t* sl, int m, int cn, int rid, int svc) {
+      const uint64_t nk = ((uint64_t)(now + svc) << 24) | (uint64_t)(uint32_t)rid;
+      const uint64_t cur = lane < cn ? sl[lane] : kKeyInf;
+      const int pos = __popc(__ballot_sync(kFull, cur < nk));
+      if (lane >= pos && lane < cn) sl[lane + 1] = cur;
+      if (lane == pos) sl[pos] = nk;
+      digest_push(W, now, call_tag(rid, m), lane);
+      if (kGeneric && lane == 0) {
+        const int recj = W->recj;
+        if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
+      }
+      __syncwarp();
+    };
+
     auto set_key = [&](int m, uint64_t nk) {
       if (lane == (m & 31)) {
         // an empty instance (nk all ones) maps to a key at or above kNoEvent
@@ -703,6 +719,27 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           if (m < 32) dirty0 = stale;
           else dirty1 = stale;
         }
+        if (kGeneric) {
+          const int recj = W->recj;
+          if (recj >= 0) {
+            const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
+            const int64_t budget = slo_budget(r->deadline - now, tail.x, tail.x + W->frest[(uint32_t)tail.w >> 24]);
+            if (lane == 0) log_dispatch(a, recj, rid, m, now, budget);
+          }
+        }
+        if (rel_count == 1) {
+          // the event's only dispatch meets an empty queue and a free slot: it
+          // starts now, as the batch boundary below would start it
+          uint64_t* const sl = W->slot + c.slot_base[m];
+          __syncwarp();
+          const int cn = W->cnt[m];
+          if (W->hsize[m] == 0 && cn < c.inst_slots[m]) {
+            start_call(sl, m, cn, rid, svc_m);
+            if (lane == 0) W->cnt[m] = cn + 1;
+            set_key(m, sl[0]);
+            continue;
+          }
+        }
         // the local-queue key is formed only if the request has to wait
         if (lane == npend) {
           pend_m = m;
@@ -713,14 +750,6 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         }
         npend++;
         touched |= 1ull << m;
-        if (kGeneric) {
-          const int recj = W->recj;
-          if (recj >= 0) {
-            const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
-            const int64_t budget = slo_budget(r->deadline - now, tail.x, tail.x + W->frest[(uint32_t)tail.w >> 24]);
-            if (lane == 0) log_dispatch(a, recj, rid, m, now, budget);
-          }
-        }
       }
 
       // Batch boundary on every touched instance: its free slots go to the most
@@ -768,19 +797,8 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             rid = top.rid;
             svc = top.svc;
           }
-          // run it until now + svc: insert its key into m's sorted slots
-          const uint64_t nk = ((uint64_t)(now + svc) << 24) | (uint64_t)(uint32_t)rid;
-          const uint64_t cur = lane < cn ? sl[lane] : kKeyInf;
-          const int pos = __popc(__ballot_sync(kFull, cur < nk));
-          if (lane >= pos && lane < cn) sl[lane + 1] = cur;
-          if (lane == pos) sl[pos] = nk;
+          start_call(sl, m, cn, rid, svc);
           ++cn;
-          digest_push(W, now, call_tag(rid, m), lane);
-          if (kGeneric && lane == 0) {
-            const int recj = W->recj;
-            if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
-          }
-          __syncwarp();
         }
         if (lane == 0) W->cnt[m] = cn;
         set_key(m, cn ? sl[0] : kKeyInf);
