@@ -434,15 +434,17 @@ __device__ __noinline__ int2 push_pop(WarpShared* W, const CallRec* rec, int64_t
 }
 
 // All lanes: a query's evaluation call finished at `now` (Sec. 4.3's metrics).
-__device__ __noinline__ void finish_query(WarpShared* W, int32_t qid, int64_t now, int64_t arrival, int64_t deadline,
-                                         int lane) {
+__device__ __forceinline__ void finish_query(WarpShared* W, int32_t qid, int64_t now, int64_t arrival,
+                                            int64_t deadline, int lane) {
   if (lane == 0) {
     W->slo_met += now <= deadline ? 1 : 0;
     W->n_done++;
     W->makespan = now;
   }
   digest_push(W, now, query_tag(qid), lane);
-  topk_insert_warp(W, now - arrival, lane);
+  // most latencies of a full heap fall below its root and change nothing
+  const int64_t v = now - arrival;
+  if (W->tk < W->kcap || v > W->tkmin) topk_insert_warp(W, v, lane);
 }
 
 __device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, int m, int64_t now, int64_t budget) {
