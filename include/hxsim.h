@@ -35,7 +35,20 @@
  *    request id / query id);
  *  - per simulation the nearest-rank P95 of query latencies
  *    (sorted L[ceil(0.95 n) - 1]), the number of queries with latency <= T_slo,
- *    T_slo = slo_mult * (S + slowest chain + E on the reference type).
+ *    T_slo = slo_mult * (S + slowest chain + E on the reference type);
+ *  - Sec. 5's further settings: several tenants, each with its own SLO
+ *    multiplier (the multi-tenant evaluation); single-shot requests, a query
+ *    of one E call with k = 0 (the competing workloads), released on
+ *    arrival, whose budget denominator is its own tbar; and instances that
+ *    become slow or unavailable for a while, handled by timeout and re-issue
+ *    (Sec. 3.3): an attempt that starts on an instance inside one of its
+ *    fault windows runs slow_fp / SCALE times longer (rounded up; 0 = never
+ *    finishes), and with a timeout factor it fails at start + timeout_mult *
+ *    its t_comp on that instance if it would run longer; the failure frees
+ *    its slot and t_queue like a completion, releases nothing, and the
+ *    request is dispatched again at that time over the other instances
+ *    (round robin steps past the failed one).  Attempts that start outside
+ *    every window never time out.
  *
  * Errors: every function returns an HX_* status; nothing throws or aborts
  * across the ABI.  hx_last_error() returns the calling thread's last message.
@@ -75,6 +88,8 @@ enum { HX_OBJ_P95 = 0, HX_OBJ_P95_SLO95 = 1 };
 #define HX_MAX_SLOTS 16
 #define HX_MAX_K 8
 #define HX_MAX_RETRY 15
+#define HX_MAX_TENANTS 4
+#define HX_MAX_FAULTS 16
 
 /* One request trace (host memory).  Calls of query i are
  * [call_base[i], call_base[i+1]) in the order S, G_0..G_{k-1}, the
@@ -84,7 +99,7 @@ typedef struct hx_trace {
   int32_t n_queries;
   int32_t n_calls;              /* < 2^24 */
   const int64_t* arrival_us;    /* [n_queries] non-decreasing, >= 0 */
-  const uint8_t* k;             /* [n_queries] 1..8 */
+  const uint8_t* k;             /* [n_queries] 1..8, or 0 for a single-shot request (one E call) */
   const int32_t* call_base;     /* [n_queries + 1] */
   const int32_t* prompt;        /* [n_calls] >= 1 */
   const int32_t* out;           /* [n_calls] true output tokens >= 0 */
@@ -92,7 +107,20 @@ typedef struct hx_trace {
   const uint8_t* stage;         /* [n_calls] HX_STAGE_* */
   const uint8_t* cand;          /* [n_calls] candidate c (G and C calls) */
   const uint8_t* retry;         /* [n_calls] r for C calls, 0 otherwise */
+  const uint8_t* tenant;        /* [n_queries] < cluster n_tenants; NULL = all tenant 0 */
 } hx_trace;
+
+/* A fault window of one instance: attempts that start on `inst` at a time in
+ * [t0_us, t1_us) run slow_fp / SCALE times longer; slow_fp = 0 means they
+ * never finish (only allowed with a timeout).  The first listed window that
+ * covers a start applies. */
+typedef struct hx_fault {
+  int32_t inst;
+  int32_t pad;
+  int64_t t0_us;                    /* 0 <= t0_us <= t1_us <= 2^38 */
+  int64_t t1_us;
+  int64_t slow_fp;                  /* 0, or SCALE / 100 .. 100 * SCALE */
+} hx_fault;
 
 /* Heterogeneous instances (Sec. 3.3's empirical performance profiles). */
 typedef struct hx_cluster {
@@ -107,6 +135,12 @@ typedef struct hx_cluster {
   int32_t rmax;                     /* workflow's retry bound R, 0..15 */
   const int32_t* stage_ref_prompt;  /* [4] reference tokens per stage (S,G,C,E) */
   const int32_t* stage_ref_out;     /* [4] */
+  int32_t n_tenants;                /* 0 or 1 = one tenant; up to HX_MAX_TENANTS */
+  int32_t n_faults;                 /* 0..HX_MAX_FAULTS */
+  const int64_t* tenant_slo_mult_fp;  /* [n_tenants] SLO multipliers (<= 16 * SCALE), NULL =
+                                         slo_mult_fp for every tenant */
+  int64_t timeout_mult_fp;          /* 0 = no timeout, else SCALE .. 100 * SCALE */
+  const hx_fault* faults;           /* [n_faults] */
 } hx_cluster;
 
 /* Hyper-parameter points (host memory). */
@@ -155,6 +189,15 @@ typedef struct hx_best {
   int32_t* per_trace_point;   /* caller-owned [n_traces], may be NULL */
 } hx_best;
 
+/* Per-simulation counts beside hx_result: SLO hits and completed queries
+ * per tenant, and the attempts that timed out and were re-issued. */
+typedef struct hx_extra {
+  int32_t slo_met[HX_MAX_TENANTS];
+  int32_t n_done[HX_MAX_TENANTS];
+  int32_t reissued;
+  int32_t pad;
+} hx_extra;
+
 typedef struct hx_sim hx_sim;
 
 /* Validate and copy traces, cluster and grid to library-owned device memory
@@ -174,6 +217,10 @@ int hx_sim_run(hx_sim* h, void* stream);
 
 /* Wait for the last run and copy n <= n_sims results to host memory. */
 int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n);
+
+/* Wait for the last run and copy n <= n_sims per-tenant counts (see
+ * hx_extra); same indexing as hx_sim_results. */
+int hx_sim_extras(hx_sim* h, hx_extra* host_out, size_t n);
 
 /* Wait for the last run and return the best point for `objective`. */
 int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out);

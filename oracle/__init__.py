@@ -21,6 +21,8 @@ _LIB = os.path.join(_HERE, "libhxoracle.so")
 RESULT_DTYPE = np.dtype([("p95_us", "<i8"), ("makespan_us", "<i8"), ("events", "<i8"),
                          ("digest", "<u8"), ("slo_met", "<i4"), ("n_done", "<i4"),
                          ("status", "<i4"), ("pad", "<i4")])
+EXTRA_DTYPE = np.dtype([("slo_met", "<i4", (4,)), ("n_done", "<i4", (4,)), ("reissued", "<i4"), ("pad", "<i4")])
+FAULT_DTYPE = np.dtype([("inst", "<i4"), ("pad", "<i4"), ("t0_us", "<i8"), ("t1_us", "<i8"), ("slow_fp", "<i8")])
 
 
 def build(force: bool = False) -> str:
@@ -38,7 +40,8 @@ class _Trace(ctypes.Structure):
     _fields_ = [("n_queries", ctypes.c_int32), ("n_calls", ctypes.c_int32),
                 ("arrival_us", ctypes.c_void_p), ("k", ctypes.c_void_p), ("call_base", ctypes.c_void_p),
                 ("prompt", ctypes.c_void_p), ("out", ctypes.c_void_p), ("out_est", ctypes.c_void_p),
-                ("stage", ctypes.c_void_p), ("cand", ctypes.c_void_p), ("retry", ctypes.c_void_p)]
+                ("stage", ctypes.c_void_p), ("cand", ctypes.c_void_p), ("retry", ctypes.c_void_p),
+                ("tenant", ctypes.c_void_p)]
 
 
 class _Cluster(ctypes.Structure):
@@ -46,7 +49,10 @@ class _Cluster(ctypes.Structure):
                 ("decode_us_tok", ctypes.c_void_p), ("slots", ctypes.c_void_p),
                 ("n_inst", ctypes.c_int32), ("inst_type", ctypes.c_void_p), ("ref_type", ctypes.c_int32),
                 ("slo_mult_fp", ctypes.c_int64), ("rmax", ctypes.c_int32),
-                ("stage_ref_prompt", ctypes.c_void_p), ("stage_ref_out", ctypes.c_void_p)]
+                ("stage_ref_prompt", ctypes.c_void_p), ("stage_ref_out", ctypes.c_void_p),
+                ("n_tenants", ctypes.c_int32), ("n_faults", ctypes.c_int32),
+                ("tenant_slo_mult_fp", ctypes.c_void_p), ("timeout_mult_fp", ctypes.c_int64),
+                ("faults", ctypes.c_void_p)]
 
 
 class _Log(ctypes.Structure):
@@ -97,13 +103,24 @@ class _Marshal:
         self.t = [_c(t.arrival_us, np.int64), _c(t.k, np.uint8), _c(t.call_base, np.int32),
                   _c(t.prompt, np.int32), _c(t.out, np.int32), _c(t.out_est, np.int32),
                   _c(t.stage, np.uint8), _c(t.cand, np.uint8), _c(t.retry, np.uint8)]
-        self.trace = _Trace(int(self.t[0].shape[0]), int(self.t[3].shape[0]), *[_ptr(a) for a in self.t])
+        ten = getattr(t, "tenant", None)
+        self.tenant = None if ten is None else _c(ten, np.uint8)
+        self.trace = _Trace(int(self.t[0].shape[0]), int(self.t[3].shape[0]), *[_ptr(a) for a in self.t],
+                            None if self.tenant is None else _ptr(self.tenant))
         c = cluster
         self.c = [_c(c.prefill_tok_s, np.int32), _c(c.decode_us_tok, np.int32), _c(c.slots, np.int32),
                   _c(c.inst_type, np.uint8), _c(c.stage_ref_prompt, np.int32), _c(c.stage_ref_out, np.int32)]
+        tm = getattr(c, "tenant_slo_mult_fp", None)
+        self.tmult = None if tm is None else _c(tm, np.int64)
+        fl = getattr(c, "faults", None)
+        self.faults = np.zeros(0, FAULT_DTYPE) if fl is None else np.ascontiguousarray(fl, dtype=FAULT_DTYPE)
         self.cluster = _Cluster(int(self.c[0].shape[0]), _ptr(self.c[0]), _ptr(self.c[1]), _ptr(self.c[2]),
                                 int(self.c[3].shape[0]), _ptr(self.c[3]), int(c.ref_type),
-                                int(c.slo_mult_fp), int(c.rmax), _ptr(self.c[4]), _ptr(self.c[5]))
+                                int(c.slo_mult_fp), int(c.rmax), _ptr(self.c[4]), _ptr(self.c[5]),
+                                1 if self.tmult is None else int(self.tmult.shape[0]), int(self.faults.shape[0]),
+                                None if self.tmult is None else _ptr(self.tmult),
+                                int(getattr(c, "timeout_mult_fp", 0)),
+                                _ptr(self.faults) if self.faults.shape[0] else None)
 
 
 def point_of(grid, p: int) -> Dict[str, int]:
@@ -131,42 +148,48 @@ def prep(trace, cluster) -> Dict[str, np.ndarray]:
                 t_slo=tslo[:nq], stage_ref_cost=cref)
 
 
-def simulate(trace, cluster, point: Dict[str, int], check: bool = False, log: bool = False):
-    """One simulation.  Returns the result record (and per-call logs if asked)."""
+def simulate(trace, cluster, point: Dict[str, int], check: bool = False, log: bool = False,
+             extra: bool = False):
+    """One simulation.  Returns the result record, then the per-call logs if
+    `log`, then the per-tenant counts and re-issues (EXTRA_DTYPE) if `extra`."""
     lib = _load()
     m = _Marshal(trace, cluster)
     pt = _Point(point["alpha_fp"], point["gamma_fp"], point["beta_us2"], point["rho"],
                 point["local_policy"], point["dispatch_policy"])
     res = np.zeros(1, RESULT_DTYPE)
+    ext = np.zeros(1, EXTRA_DTYPE)
     if not log:
         lib.hxo_simulate(ctypes.byref(m.trace), ctypes.byref(m.cluster), ctypes.byref(pt), int(check),
-                         _ptr(res), None)
-        return res[0]
+                         _ptr(res), None, _ptr(ext))
+        return (res[0], ext[0]) if extra else res[0]
     nc = max(trace.n_calls, 1)
     arrs = dict(inst=np.full(nc, -1, np.int32), enq=np.full(nc, -1, np.int64),
                 budget=np.zeros(nc, np.int64), start=np.full(nc, -1, np.int64),
                 end=np.full(nc, -1, np.int64))
     lg = _Log(*[_ptr(arrs[k]) for k in ("inst", "enq", "budget", "start", "end")])
     lib.hxo_simulate(ctypes.byref(m.trace), ctypes.byref(m.cluster), ctypes.byref(pt), int(check),
-                     _ptr(res), ctypes.byref(lg))
+                     _ptr(res), ctypes.byref(lg), _ptr(ext))
     n = trace.n_calls
-    return res[0], {k: v[:n] for k, v in arrs.items()}
+    logs = {k: v[:n] for k, v in arrs.items()}
+    return (res[0], logs, ext[0]) if extra else (res[0], logs)
 
 
 def _run_one(args):
-    trace, cluster, point, check = args
-    return simulate(trace, cluster, point, check=check)
+    trace, cluster, point, check, extra = args
+    return simulate(trace, cluster, point, check=check, extra=extra)
 
 
-def run(workload, sims: Optional[Sequence[int]] = None, procs: int = 1, check: bool = False) -> np.ndarray:
-    """Simulate the listed sims (index = trace * P + point) of a workload.
+def run(workload, sims: Optional[Sequence[int]] = None, procs: int = 1, check: bool = False,
+        extra: bool = False):
+    """Simulate the listed sims (index = trace * P + point) of a workload;
+    with `extra`, also return their per-tenant counts (EXTRA_DTYPE).
 
     With procs > 1 the sims run in a process pool started with `spawn`.
     """
     P = workload.grid.n_points
     if sims is None:
         sims = range(len(workload.traces) * P)
-    jobs = [(workload.traces[s // P], workload.cluster, point_of(workload.grid, s % P), check) for s in sims]
+    jobs = [(workload.traces[s // P], workload.cluster, point_of(workload.grid, s % P), check, extra) for s in sims]
     if procs <= 1 or len(jobs) <= 1:
         out = [_run_one(j) for j in jobs]
     else:
@@ -175,9 +198,13 @@ def run(workload, sims: Optional[Sequence[int]] = None, procs: int = 1, check: b
         with ctx.Pool(procs) as pool:
             out = pool.map(_run_one, jobs, chunksize=max(1, len(jobs) // (4 * procs)))
     res = np.zeros(len(jobs), RESULT_DTYPE)
+    ext = np.zeros(len(jobs), EXTRA_DTYPE)
     for i, r in enumerate(out):
-        res[i] = r
-    return res
+        if extra:
+            res[i], ext[i] = r
+        else:
+            res[i] = r
+    return (res, ext) if extra else res
 
 
 def budget(t_slo: int, elapsed: int, tbar: int, remaining: int) -> int:

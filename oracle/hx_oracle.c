@@ -31,7 +31,26 @@
  *    arrivals, instance, request id / query id); after each event the
  *    released successors are dispatched in request-id order, then every
  *    instance with a free slot starts its most urgent waiting request;
- *  - P95 is the nearest-rank percentile: sorted latencies L[ceil(.95 n) - 1].
+ *  - P95 is the nearest-rank percentile: sorted latencies L[ceil(.95 n) - 1];
+ *  - several tenants (the multi-tenant evaluation of Sec. 5): each query
+ *    belongs to one, whose SLO multiplier replaces the cluster's in T_slo;
+ *    SLO attainment is also counted per tenant;
+ *  - a single-shot request (the competing workloads of Sec. 5) is a query
+ *    with k = 0 made of one evaluation-stage call E: it is dispatched on
+ *    arrival, its budget denominator is its own mean cost and its exclusive
+ *    latency is that call on the reference type;
+ *  - timeout and re-issue (Sec. 3.3, for an instance that becomes slow or
+ *    unavailable): an attempt that starts on an instance inside one of its
+ *    fault windows runs slow_fp / SCALE times longer (rounded up; slow_fp =
+ *    0: it never finishes; the first listed window that covers the start
+ *    applies).  With a timeout factor, such an attempt whose running time
+ *    would exceed timeout_mult * its Eq. (comp) estimate on that instance
+ *    fails at start + that timeout (attempts started outside every window
+ *    never time out, so re-issues end with the windows): like a completion it
+ *    frees its slot and its estimate from Theta^m, releases nothing, and
+ *    the request is dispatched again at that time by the same policy over
+ *    the other instances (over all of them when there is one); round robin
+ *    steps past the failed instance.  Per-call logs keep the last attempt.
  */
 #include "hx_oracle.h"
 
@@ -106,11 +125,24 @@ static int validate(const hxo_trace* tr, const hxo_cluster* cl) {
   for (int m = 0; m < cl->n_inst; ++m)
     if (cl->inst_type[m] >= cl->n_types) return 0;
   if (cl->ref_type < 0 || cl->ref_type >= cl->n_types || cl->rmax < 0) return 0;
+  if (cl->n_tenants < 1 || cl->n_tenants > HXO_MAX_TENANTS || cl->n_faults < 0) return 0;
+  if (cl->timeout_mult_fp != 0 && cl->timeout_mult_fp < FP_ONE) return 0;
+  for (int f = 0; f < cl->n_faults; ++f) {
+    const hxo_fault* F = &cl->faults[f];
+    if (F->inst < 0 || F->inst >= cl->n_inst || F->t0_us < 0 || F->t1_us < F->t0_us || F->slow_fp < 0) return 0;
+    if (F->slow_fp == 0 && cl->timeout_mult_fp == 0) return 0; /* would never finish */
+  }
   if (tr->n_queries < 0 || tr->call_base[0] != 0 || tr->call_base[tr->n_queries] != tr->n_calls) return 0;
   for (int32_t i = 0; i < tr->n_queries; ++i) {
     if (i > 0 && tr->arrival_us[i] < tr->arrival_us[i - 1]) return 0;
     if (tr->arrival_us[i] < 0) return 0;
+    if (tr->tenant && tr->tenant[i] >= cl->n_tenants) return 0;
     int32_t b = tr->call_base[i], e = tr->call_base[i + 1], k = tr->k[i];
+    if (k == 0) {
+      /* a single-shot request: one evaluation-stage call */
+      if (e - b != 1 || tr->stage[b] != ST_E || tr->prompt[b] < 1 || tr->out[b] < 0 || tr->out_est[b] < 0) return 0;
+      continue;
+    }
     if (k < 1 || e - b < 2 + k) return 0;
     if (tr->stage[b] != ST_S || tr->stage[e - 1] != ST_E) return 0;
     for (int c = 0; c < k; ++c)
@@ -192,7 +224,9 @@ int hxo_prep(const hxo_trace* tr, const hxo_cluster* cl, int64_t* est, int64_t* 
     for (int c = 0; c < tr->k[i]; ++c)
       if (chain[c] > longest) longest = chain[c];
     int64_t l0 = l_s + longest + l_e;
-    t_slo[i] = (int64_t)(((i128)cl->slo_mult_fp * l0) / FP_ONE);
+    int64_t mult = cl->slo_mult_fp;
+    if (cl->tenant_slo_mult_fp) mult = cl->tenant_slo_mult_fp[tr->tenant ? tr->tenant[i] : 0];
+    t_slo[i] = (int64_t)(((i128)mult * l0) / FP_ONE);
   }
   return HXO_OK;
 }
@@ -238,8 +272,10 @@ typedef struct {
   int64_t* q;           /* per instance: sum of Eq. (comp) over Theta^m */
   ivec* waiting;        /* per instance */
   ivec* running;        /* per instance */
+  uint8_t* failed;      /* per call: the running attempt times out */
   int64_t rr_next;
   uint64_t digest;
+  int32_t reissued;
   int bad;
 } sim_t;
 
@@ -265,9 +301,10 @@ static int64_t remaining_cost(const sim_t* s, int32_t c, int64_t tb) {
   }
 }
 
-/* Global coordinator (Sec. 4.1): budget at send time, score every instance,
- * dispatch to the highest score (lowest index on ties), enqueue there. */
-static void dispatch(sim_t* s, int32_t c, int64_t now) {
+/* Global coordinator (Sec. 4.1): budget at send time, score every instance
+ * but `excl` (a re-issue's failed instance, -1 for none), dispatch to the
+ * highest score (lowest index on ties), enqueue there. */
+static void dispatch(sim_t* s, int32_t c, int64_t now, int excl) {
   const hxo_trace* tr = s->tr;
   const hxo_cluster* cl = s->cl;
   int32_t i = s->qid[c];
@@ -276,12 +313,18 @@ static void dispatch(sim_t* s, int32_t c, int64_t now) {
   s->remaining[c] = remaining_cost(s, c, tb);
   s->budget[c] = hxo_budget(s->t_slo[i], elapsed, tb, s->remaining[c]);
   int best = -1;
+  if (cl->n_inst == 1) excl = -1;
   if (s->pt->dispatch_policy == 1) {
     best = (int)(s->rr_next % cl->n_inst);
     s->rr_next++;
+    if (best == excl) {
+      best = (int)(s->rr_next % cl->n_inst);
+      s->rr_next++;
+    }
   } else {
     int64_t best_score = 0;
     for (int m = 0; m < cl->n_inst; ++m) {
+      if (m == excl) continue;
       int64_t sc = hxo_score(s->pt->alpha_fp, s->pt->beta_us2, s->q[m], est_on(tr, cl, m, c));
       if (best < 0 || sc > best_score) {
         best = m;
@@ -294,6 +337,32 @@ static void dispatch(sim_t* s, int32_t c, int64_t now) {
   s->state[c] = C_WAITING;
   s->q[best] += est_on(tr, cl, best, c);
   if (!ivec_push(&s->waiting[best], c)) s->bad = HXO_ERR_OOM;
+}
+
+/* Running time of an attempt of call c started on m at `now` under the
+ * cluster's fault windows and timeout; *fail says the attempt times out. */
+static int64_t attempt_time(const sim_t* s, int m, int32_t c, int64_t now, int* fail) {
+  const hxo_cluster* cl = s->cl;
+  int64_t run = svc_on(s->tr, cl, m, c);
+  int in_window = 0, down = 0;
+  for (int f = 0; f < cl->n_faults; ++f) {
+    const hxo_fault* F = &cl->faults[f];
+    if (F->inst == m && now >= F->t0_us && now < F->t1_us) {
+      in_window = 1;
+      if (F->slow_fp == 0) down = 1;
+      else run = (int64_t)(((i128)run * F->slow_fp + FP_ONE - 1) / FP_ONE);
+      break;
+    }
+  }
+  *fail = 0;
+  if (in_window && cl->timeout_mult_fp > 0) {
+    int64_t timeout = (int64_t)(((i128)est_on(s->tr, cl, m, c) * cl->timeout_mult_fp) / FP_ONE);
+    if (down || run > timeout) {
+      *fail = 1;
+      return timeout;
+    }
+  }
+  return run;
 }
 
 /* Local queues (Sec. 4.2): at a batch boundary each instance with a free slot
@@ -335,7 +404,9 @@ static void fill_slots(sim_t* s, int64_t now, int64_t** ubuf, int64_t** ebuf, in
       if (!ivec_push(&s->running[m], c)) { s->bad = HXO_ERR_OOM; return; }
       s->state[c] = C_RUNNING;
       s->start[c] = now;
-      s->end[c] = now + svc_on(tr, cl, m, c);
+      int fail;
+      s->end[c] = now + attempt_time(s, m, c, now, &fail);
+      s->failed[c] = (uint8_t)fail;
       s->digest += call_term(c, m, now);
     }
   }
@@ -356,8 +427,9 @@ static int check_invariants(const sim_t* s) {
 }
 
 int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt, int check,
-                 hxo_result* res, const hxo_log* log) {
+                 hxo_result* res, const hxo_log* log, hxo_extra* ext) {
   memset(res, 0, sizeof(*res));
+  if (ext) memset(ext, 0, sizeof(*ext));
   res->p95_us = -1;
   if (!validate(tr, cl) || pt->alpha_fp < 0 || pt->alpha_fp > FP_ONE || pt->beta_us2 < 0 ||
       pt->gamma_fp < 0 || pt->rho < 0 || pt->local_policy < 0 || pt->local_policy > 2 ||
@@ -382,6 +454,7 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
   s.remaining = (int64_t*)calloc(nc1, sizeof(int64_t));
   s.start = (int64_t*)calloc(nc1, sizeof(int64_t));
   s.end = (int64_t*)calloc(nc1, sizeof(int64_t));
+  s.failed = (uint8_t*)calloc(nc1, 1);
   s.q = (int64_t*)calloc((size_t)N, sizeof(int64_t));
   s.waiting = (ivec*)calloc((size_t)N, sizeof(ivec));
   s.running = (ivec*)calloc((size_t)N, sizeof(ivec));
@@ -394,7 +467,7 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
   int32_t bufcap = 0;
   int status = HXO_OK;
   if (!s.t_slo || !s.chains_left || !s.qid || !s.state || !s.inst || !s.enq || !s.budget || !s.remaining || !s.start ||
-      !s.end || !s.q || !s.waiting || !s.running || !lat || !est_tmp || !svc_tmp || !tbar_tmp) {
+      !s.end || !s.failed || !s.q || !s.waiting || !s.running || !lat || !est_tmp || !svc_tmp || !tbar_tmp) {
     status = HXO_ERR_OOM;
     goto done;
   }
@@ -403,6 +476,7 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
     for (int32_t j = tr->call_base[i]; j < tr->call_base[i + 1]; ++j) s.qid[j] = i;
 
   int32_t next_q = 0, n_done = 0, slo_met = 0;
+  int32_t t_slo_met[HXO_MAX_TENANTS] = {0, 0, 0, 0}, t_done[HXO_MAX_TENANTS] = {0, 0, 0, 0};
   int64_t makespan = 0, events = 0;
   for (;;) {
     /* next event: earliest completion by (end, instance, rid), else arrival */
@@ -427,8 +501,18 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
       now = s.end[c];
       for (int32_t j = 0; j < s.running[m].n; ++j)
         if (s.running[m].v[j] == c) { ivec_remove_at(&s.running[m], j); break; }
-      s.state[c] = C_DONE;
       s.q[m] -= est_on(tr, cl, m, c);
+      if (s.failed[c]) {
+        /* the attempt timed out: the request goes out again, not to m */
+        s.failed[c] = 0;
+        s.reissued++;
+        dispatch(&s, c, now, m);
+        fill_slots(&s, now, &ubuf, &ebuf, &rbuf, &bufcap);
+        if (s.bad) { status = s.bad; goto done; }
+        if (check && !check_invariants(&s)) { status = HXO_ERR_INVARIANT; goto done; }
+        continue;
+      }
+      s.state[c] = C_DONE;
       events++;
       int32_t i = s.qid[c];
       int32_t b = tr->call_base[i], e = tr->call_base[i + 1];
@@ -436,28 +520,33 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
       if (st == ST_S) {
         s.chains_left[i] = tr->k[i];
         for (int32_t j = b; j < e; ++j)
-          if (tr->stage[j] == ST_G) dispatch(&s, j, now);
+          if (tr->stage[j] == ST_G) dispatch(&s, j, now, -1);
       } else if (st == ST_G || st == ST_C) {
         int cand = tr->cand[c], r_next = (st == ST_G ? 0 : tr->retry[c]) + 1;
         int32_t nxt = -1;
         for (int32_t j = b; j < e; ++j)
           if (tr->stage[j] == ST_C && tr->cand[j] == cand && tr->retry[j] == r_next) nxt = j;
         if (nxt >= 0) {
-          dispatch(&s, nxt, now);
+          dispatch(&s, nxt, now, -1);
         } else if (--s.chains_left[i] == 0) {
           for (int32_t j = b; j < e; ++j)
-            if (tr->stage[j] == ST_E) dispatch(&s, j, now);
+            if (tr->stage[j] == ST_E) dispatch(&s, j, now, -1);
         }
       } else {
         int64_t l = now - tr->arrival_us[i];
+        int ten = tr->tenant ? tr->tenant[i] : 0;
         lat[n_done++] = l;
-        if (l <= s.t_slo[i]) slo_met++;
+        t_done[ten]++;
+        if (l <= s.t_slo[i]) {
+          slo_met++;
+          t_slo_met[ten]++;
+        }
         if (now > makespan) makespan = now;
         s.digest += query_term(i, now);
       }
     } else {
       now = tr->arrival_us[next_q];
-      dispatch(&s, tr->call_base[next_q], now);
+      dispatch(&s, tr->call_base[next_q], now, -1);
       next_q++;
     }
     fill_slots(&s, now, &ubuf, &ebuf, &rbuf, &bufcap);
@@ -472,6 +561,13 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
 
   res->n_done = n_done;
   res->slo_met = slo_met;
+  if (ext) {
+    for (int t = 0; t < HXO_MAX_TENANTS; ++t) {
+      ext->slo_met[t] = t_slo_met[t];
+      ext->n_done[t] = t_done[t];
+    }
+    ext->reissued = s.reissued;
+  }
   res->makespan_us = makespan;
   res->events = events;
   res->digest = s.digest;
@@ -500,7 +596,7 @@ done:
   if (s.running)
     for (int m = 0; m < N; ++m) free(s.running[m].v);
   free(s.t_slo); free(s.chains_left); free(s.qid); free(s.state); free(s.inst); free(s.enq);
-  free(s.budget); free(s.remaining); free(s.start); free(s.end); free(s.q); free(s.waiting); free(s.running);
+  free(s.budget); free(s.remaining); free(s.start); free(s.end); free(s.failed); free(s.q); free(s.waiting); free(s.running);
   free(lat); free(est_tmp); free(svc_tmp); free(tbar_tmp); free(ubuf); free(ebuf); free(rbuf);
   return status;
 }

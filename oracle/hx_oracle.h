@@ -29,7 +29,20 @@ typedef struct {
   const uint8_t* stage;       /* [n_calls] 0=S 1=G 2=C 3=E */
   const uint8_t* cand;        /* [n_calls] */
   const uint8_t* retry;       /* [n_calls] */
+  const uint8_t* tenant;      /* [n_queries] tenant of each query, NULL = all tenant 0 */
 } hxo_trace;
+
+/* A fault window of one instance: attempts that start on it in [t0, t1)
+ * run slow_fp / SCALE times longer; slow_fp = 0 means they never finish. */
+typedef struct {
+  int32_t inst;
+  int32_t pad;
+  int64_t t0_us;
+  int64_t t1_us;
+  int64_t slow_fp;
+} hxo_fault;
+
+#define HXO_MAX_TENANTS 4
 
 typedef struct {
   int32_t n_types;
@@ -43,6 +56,11 @@ typedef struct {
   int32_t rmax;
   const int32_t* stage_ref_prompt;  /* [4] */
   const int32_t* stage_ref_out;     /* [4] */
+  int32_t n_tenants;                /* 1..HXO_MAX_TENANTS */
+  int32_t n_faults;
+  const int64_t* tenant_slo_mult_fp;  /* [n_tenants], NULL = slo_mult_fp for every tenant */
+  int64_t timeout_mult_fp;          /* 0 = no timeout, else >= SCALE */
+  const hxo_fault* faults;          /* [n_faults] */
 } hxo_cluster;
 
 typedef struct {
@@ -67,6 +85,14 @@ typedef struct {
 
 enum { HXO_OK = 0, HXO_ERR_INVALID = 1, HXO_ERR_OOM = 3, HXO_ERR_INVARIANT = 7 };
 
+/* Per-tenant SLO counts and the number of timed-out attempts re-issued. */
+typedef struct {
+  int32_t slo_met[HXO_MAX_TENANTS];
+  int32_t n_done[HXO_MAX_TENANTS];
+  int32_t reissued;
+  int32_t pad;
+} hxo_extra;
+
 /* Per-call estimates of Eq. (comp) and the mean over instances, and the
  * per-query SLO.  est/svc are [n_calls * n_types] (type-minor). */
 int hxo_prep(const hxo_trace* tr, const hxo_cluster* cl, int64_t* est, int64_t* svc,
@@ -81,10 +107,10 @@ typedef struct {
   int64_t* end;
 } hxo_log;
 
-/* One simulation.  log may be NULL.  check != 0 re-verifies the scheduler
- * invariants after every event (slow). */
+/* One simulation.  log and ext may be NULL.  check != 0 re-verifies the
+ * scheduler invariants after every event (slow). */
 int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt,
-                 int check, hxo_result* res, const hxo_log* log);
+                 int check, hxo_result* res, const hxo_log* log, hxo_extra* ext);
 
 /* SLO budget of Sec. 4.2: (T_slo - elapsed) * tbar / remaining, truncated. */
 int64_t hxo_budget(int64_t t_slo, int64_t elapsed, int64_t tbar, int64_t remaining);

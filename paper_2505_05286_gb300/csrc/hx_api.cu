@@ -44,6 +44,8 @@ struct hx_sim {
   int64_t n_sims = 0, n_q = 0, n_c = 0;
   int32_t max_nq = 0, max_nc = 0, max_kcap = 1;
   hx::ClusterK ck{};
+  int32_t n_tenants = 0;          // as given in hx_cluster (validation of later uploads)
+  std::vector<hx_fault> faults;
   std::vector<int32_t> h_nq, h_nc;
   // device: inputs
   int64_t* d_arrival = nullptr;
@@ -51,6 +53,7 @@ struct hx_sim {
   int64_t* d_q_off = nullptr;
   int64_t* d_c_off = nullptr;
   uint8_t* d_k = nullptr;
+  uint8_t* d_tenant = nullptr;
   int32_t* d_prompt = nullptr;
   int32_t* d_out = nullptr;
   int32_t* d_out_est = nullptr;
@@ -66,6 +69,7 @@ struct hx_sim {
   // device: derived and outputs
   hx::CallRec* d_rec = nullptr;
   hx_result* d_results = nullptr;
+  hx_extra* d_extras = nullptr;  // generic kernel only
   unsigned long long* d_counter = nullptr;
   hx::BestCand* d_best_trace = nullptr;
   hx::BestCand* d_best_global = nullptr;
@@ -143,6 +147,25 @@ int validate_cluster(const hx_cluster* c, int64_t* min_prefill, int64_t* max_dec
     if (p < 0 || p > kTokMax || o < 0 || o > kTokMax) return fail(HX_ERR_INVALID, "stage reference tokens out of range");
     if ((p * 1000000 + mp - 1) / mp + o * md >= kCostMax) return fail(HX_ERR_INVALID, "stage reference cost too large");
   }
+  if (c->n_tenants < 0 || c->n_tenants > HX_MAX_TENANTS) return fail(HX_ERR_INVALID, "n_tenants must be 0..4");
+  if (c->tenant_slo_mult_fp)
+    for (int t = 0; t < std::max(c->n_tenants, 1); ++t)
+      if (c->tenant_slo_mult_fp[t] < 0 || c->tenant_slo_mult_fp[t] > 16 * HX_SCALE)
+        return fail(HX_ERR_INVALID, "tenant_slo_mult_fp must be 0..16*SCALE");
+  if (c->timeout_mult_fp != 0 && (c->timeout_mult_fp < HX_SCALE || c->timeout_mult_fp > 100 * HX_SCALE))
+    return fail(HX_ERR_INVALID, "timeout_mult_fp must be 0 or SCALE..100*SCALE");
+  if (c->n_faults < 0 || c->n_faults > HX_MAX_FAULTS) return fail(HX_ERR_INVALID, "n_faults must be 0..16");
+  if (c->n_faults > 0 && !c->faults) return fail(HX_ERR_INVALID, "faults is NULL");
+  for (int f = 0; f < c->n_faults; ++f) {
+    const hx_fault& F = c->faults[f];
+    if (F.inst < 0 || F.inst >= c->n_inst) return fail(HX_ERR_INVALID, "fault instance out of range");
+    if (F.t0_us < 0 || F.t1_us < F.t0_us || F.t1_us > (int64_t(1) << 38))
+      return fail(HX_ERR_INVALID, "fault window must satisfy 0 <= t0 <= t1 <= 2^38");
+    if (F.slow_fp != 0 && (F.slow_fp < HX_SCALE / 100 || F.slow_fp > 100 * HX_SCALE))
+      return fail(HX_ERR_INVALID, "fault slow_fp must be 0 or SCALE/100..100*SCALE");
+    if (F.slow_fp == 0 && c->timeout_mult_fp == 0)
+      return fail(HX_ERR_INVALID, "a stopped instance (slow_fp = 0) needs a timeout");
+  }
   *min_prefill = mp;
   *max_decode = md;
   return HX_OK;
@@ -179,22 +202,30 @@ int validate_trace(const hx_trace* tr, int ti, const hx_cluster* c, int64_t min_
       return fail(HX_ERR_INVALID, where + "arrivals must be non-negative and sorted");
     const int32_t b = tr->call_base[i], e = tr->call_base[i + 1];
     const int k = tr->k[i];
-    if (k < 1 || k > HX_MAX_K) return fail(HX_ERR_INVALID, where + "k must be 1..8");
-    if (e - b < 2 + k || b < 0 || e > tr->n_calls) return fail(HX_ERR_INVALID, where + "bad call_base");
-    if (tr->stage[b] != HX_STAGE_S || tr->stage[e - 1] != HX_STAGE_E)
-      return fail(HX_ERR_INVALID, where + "a query must start with S and end with E");
-    for (int cd = 0; cd < k; ++cd)
-      if (tr->stage[b + 1 + cd] != HX_STAGE_G || tr->cand[b + 1 + cd] != cd)
-        return fail(HX_ERR_INVALID, where + "S must be followed by G_0..G_{k-1}");
-    int prev_c = -1, prev_r = 0;
-    for (int32_t j = b + 1 + k; j < e - 1; ++j) {
-      const int cd = tr->cand[j], r = tr->retry[j];
-      if (tr->stage[j] != HX_STAGE_C || cd >= k || r < 1 || r > c->rmax)
-        return fail(HX_ERR_INVALID, where + "corrections must be C calls of a candidate with 1 <= retry <= rmax");
-      if (cd == prev_c ? r != prev_r + 1 : (cd < prev_c || r != 1))
-        return fail(HX_ERR_INVALID, where + "corrections must be ordered by (candidate, retry)");
-      prev_c = cd;
-      prev_r = r;
+    if (tr->tenant && tr->tenant[i] >= std::max(c->n_tenants, 1))
+      return fail(HX_ERR_INVALID, where + "tenant out of range");
+    if (k == 0) {
+      // a single-shot request: one evaluation-stage call
+      if (e - b != 1 || b < 0 || e > tr->n_calls || tr->stage[b] != HX_STAGE_E)
+        return fail(HX_ERR_INVALID, where + "a k = 0 query must be a single E call");
+    } else {
+      if (k > HX_MAX_K) return fail(HX_ERR_INVALID, where + "k must be 0..8");
+      if (e - b < 2 + k || b < 0 || e > tr->n_calls) return fail(HX_ERR_INVALID, where + "bad call_base");
+      if (tr->stage[b] != HX_STAGE_S || tr->stage[e - 1] != HX_STAGE_E)
+        return fail(HX_ERR_INVALID, where + "a query must start with S and end with E");
+      for (int cd = 0; cd < k; ++cd)
+        if (tr->stage[b + 1 + cd] != HX_STAGE_G || tr->cand[b + 1 + cd] != cd)
+          return fail(HX_ERR_INVALID, where + "S must be followed by G_0..G_{k-1}");
+      int prev_c = -1, prev_r = 0;
+      for (int32_t j = b + 1 + k; j < e - 1; ++j) {
+        const int cd = tr->cand[j], r = tr->retry[j];
+        if (tr->stage[j] != HX_STAGE_C || cd >= k || r < 1 || r > c->rmax)
+          return fail(HX_ERR_INVALID, where + "corrections must be C calls of a candidate with 1 <= retry <= rmax");
+        if (cd == prev_c ? r != prev_r + 1 : (cd < prev_c || r != 1))
+          return fail(HX_ERR_INVALID, where + "corrections must be ordered by (candidate, retry)");
+        prev_c = cd;
+        prev_r = r;
+      }
     }
     for (int32_t j = b; j < e; ++j) {
       const int64_t p = tr->prompt[j], o = tr->out[j], oe = tr->out_est[j];
@@ -205,7 +236,14 @@ int validate_trace(const hx_trace* tr, int ti, const hx_cluster* c, int64_t min_
       horizon += bound;
     }
   }
-  if (tr->n_queries > 0) horizon += tr->arrival_us[tr->n_queries - 1];
+  // fault windows stretch attempts (slow-down or timeout) and delay the rest
+  int64_t stretch = HX_SCALE, last = tr->n_queries > 0 ? tr->arrival_us[tr->n_queries - 1] : 0;
+  for (int f = 0; f < c->n_faults; ++f) {
+    stretch = std::max(stretch, std::max<int64_t>(c->faults[f].slow_fp, c->timeout_mult_fp));
+    last = std::max(last, c->faults[f].t1_us);
+  }
+  if (horizon > kHorizonMax) return fail(HX_ERR_INVALID, where + "time horizon exceeds 2^39 us");
+  horizon = horizon * (1 + (stretch + HX_SCALE - 1) / HX_SCALE) / (c->n_faults > 0 ? 1 : 2) + last;
   if (horizon > kHorizonMax) return fail(HX_ERR_INVALID, where + "time horizon exceeds 2^39 us");
   return HX_OK;
 }
@@ -220,7 +258,7 @@ int upload(T* dst, const T* src, int64_t count, cudaStream_t s) {
 // Copies the per-call and per-query trace arrays of all traces to the device.
 int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
   std::vector<int64_t> arrival((size_t)h->n_q), qcall((size_t)h->n_q + 1);
-  std::vector<uint8_t> kq((size_t)h->n_q);
+  std::vector<uint8_t> kq((size_t)h->n_q), tenant((size_t)h->n_q, 0);
   int64_t qo = 0, co = 0;
   for (int t = 0; t < h->n_traces; ++t) {
     const hx_trace& tr = traces[t];
@@ -228,6 +266,7 @@ int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
       arrival[qo + i] = tr.arrival_us[i];
       kq[qo + i] = tr.k[i];
       qcall[qo + i] = co + tr.call_base[i];
+      if (tr.tenant) tenant[qo + i] = tr.tenant[i];
     }
     qo += tr.n_queries;
     co += tr.n_calls;
@@ -235,7 +274,7 @@ int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
   qcall[h->n_q] = co;
   int rc;
   if ((rc = upload(h->d_arrival, arrival.data(), h->n_q, s)) || (rc = upload(h->d_k, kq.data(), h->n_q, s)) ||
-      (rc = upload(h->d_qcall, qcall.data(), h->n_q + 1, s)))
+      (rc = upload(h->d_tenant, tenant.data(), h->n_q, s)) || (rc = upload(h->d_qcall, qcall.data(), h->n_q + 1, s)))
     return rc;
   co = 0;
   for (int t = 0; t < h->n_traces; ++t) {
@@ -252,9 +291,60 @@ int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
   return HX_OK;
 }
 
-// WarpShared with its trailing slot array sized for the cluster
-int per_warp_smem(int total_slots) {
-  return (int)align_up((int64_t)offsetof(hx::WarpShared, slot) + 8 * (int64_t)std::max(total_slots, 1), 16);
+// WarpShared with its trailing slot array sized for the cluster (and one
+// fail flag per slot when the cluster has fault windows)
+int per_warp_smem(int total_slots, bool faults) {
+  const int64_t ts = std::max(total_slots, 1);
+  return (int)align_up((int64_t)offsetof(hx::WarpShared, slot) + 8 * ts + (faults ? ts : 0), 16);
+}
+
+// Kernel-parameter copy of a validated cluster.
+void fill_cluster(const hx_cluster* cluster, hx::ClusterK& ck) {
+  ck = hx::ClusterK{};
+  ck.n_inst = cluster->n_inst;
+  ck.n_types = cluster->n_types;
+  ck.ref_type = cluster->ref_type;
+  ck.rmax = cluster->rmax;
+  ck.slo_mult_fp = cluster->slo_mult_fp;
+  for (int t = 0; t < HX_MAX_TYPES; ++t) {
+    const bool on = t < cluster->n_types;
+    ck.prefill[t] = on ? cluster->prefill_tok_s[t] : 1;
+    ck.decode[t] = on ? cluster->decode_us_tok[t] : 0;
+    ck.slots[t] = on ? cluster->slots[t] : 0;
+    ck.cnt[t] = 0;
+  }
+  for (int s = 0; s < 4; ++s) {
+    ck.ref_prompt[s] = cluster->stage_ref_prompt[s];
+    ck.ref_out[s] = cluster->stage_ref_out[s];
+  }
+  int base = 0;
+  for (int m = 0; m < HX_MAX_INST; ++m) {
+    const bool on = m < cluster->n_inst;
+    const int ty = on ? cluster->inst_type[m] : 0;
+    ck.inst_type[m] = (uint8_t)ty;
+    ck.inst_slots[m] = on ? (uint8_t)cluster->slots[ty] : 0;
+    ck.slot_base[m] = (uint16_t)base;
+    if (on) {
+      base += cluster->slots[ty];
+      ck.cnt[ty]++;
+    }
+  }
+  ck.total_slots = base;
+  // per-tenant SLO multipliers replace slo_mult_fp when given
+  ck.n_tenants = cluster->tenant_slo_mult_fp ? std::max(cluster->n_tenants, 1) : 0;
+  for (int t = 0; t < HX_MAX_TENANTS; ++t)
+    ck.tenant_mult[t] = t < ck.n_tenants ? cluster->tenant_slo_mult_fp[t] : cluster->slo_mult_fp;
+  ck.timeout_mult_fp = cluster->timeout_mult_fp;
+  ck.n_faults = cluster->n_faults;
+  for (int f = 0; f < cluster->n_faults; ++f) {
+    const hx_fault& F = cluster->faults[f];
+    ck.faults[f].t0 = F.t0_us;
+    ck.faults[f].t1 = F.t1_us;
+    ck.faults[f].slow = F.slow_fp;
+    ck.faults[f].inst = F.inst;
+    ck.faults[f].pad = 0;
+  }
+  ck.smem_per_warp = per_warp_smem(base, cluster->n_faults > 0);
 }
 
 }  // namespace
@@ -303,36 +393,9 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
 
   // cluster constants (kernel parameter)
   hx::ClusterK& ck = h->ck;
-  ck.n_inst = cluster->n_inst;
-  ck.n_types = cluster->n_types;
-  ck.ref_type = cluster->ref_type;
-  ck.rmax = cluster->rmax;
-  ck.slo_mult_fp = cluster->slo_mult_fp;
-  for (int t = 0; t < HX_MAX_TYPES; ++t) {
-    const bool on = t < cluster->n_types;
-    ck.prefill[t] = on ? cluster->prefill_tok_s[t] : 1;
-    ck.decode[t] = on ? cluster->decode_us_tok[t] : 0;
-    ck.slots[t] = on ? cluster->slots[t] : 0;
-    ck.cnt[t] = 0;
-  }
-  for (int s = 0; s < 4; ++s) {
-    ck.ref_prompt[s] = cluster->stage_ref_prompt[s];
-    ck.ref_out[s] = cluster->stage_ref_out[s];
-  }
-  int base = 0;
-  for (int m = 0; m < HX_MAX_INST; ++m) {
-    const bool on = m < cluster->n_inst;
-    const int ty = on ? cluster->inst_type[m] : 0;
-    ck.inst_type[m] = (uint8_t)ty;
-    ck.inst_slots[m] = on ? (uint8_t)cluster->slots[ty] : 0;
-    ck.slot_base[m] = (uint16_t)base;
-    if (on) {
-      base += cluster->slots[ty];
-      ck.cnt[ty]++;
-    }
-  }
-  ck.total_slots = base;
-  ck.smem_per_warp = per_warp_smem(base);
+  fill_cluster(cluster, ck);
+  h->n_tenants = cluster->n_tenants;
+  h->faults.assign(cluster->faults, cluster->faults + cluster->n_faults);
 
   int dev = 0;
   cudaDeviceProp prop;
@@ -342,6 +405,7 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   }
   // device inputs
   if ((rc = h->alloc(&h->d_arrival, h->n_q)) || (rc = h->alloc(&h->d_k, h->n_q)) ||
+      (rc = h->alloc(&h->d_tenant, h->n_q)) ||
       (rc = h->alloc(&h->d_qcall, h->n_q + 1)) || (rc = h->alloc(&h->d_q_off, n_traces + 1)) ||
       (rc = h->alloc(&h->d_c_off, n_traces + 1)) || (rc = h->alloc(&h->d_prompt, h->n_c)) ||
       (rc = h->alloc(&h->d_out, h->n_c)) || (rc = h->alloc(&h->d_out_est, h->n_c)) ||
@@ -365,8 +429,9 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
     return bail(rc);
 
   // the lean instantiation serves grids that are all workload-balanced
-  // dispatch with the urgency queue and log nothing
-  h->generic = (opt && (opt->n_record > 0 || opt->force_generic));
+  // dispatch with the urgency queue, log nothing, count one tenant and have
+  // no fault windows
+  h->generic = (opt && (opt->n_record > 0 || opt->force_generic)) || ck.n_tenants > 1 || ck.n_faults > 0;
   for (int p = 0; p < grid->n_points && !h->generic; ++p)
     if (grid->local_policy[p] != HX_LOCAL_PQ || grid->dispatch_policy[p] != HX_DISPATCH_WB) h->generic = true;
   const void* kfn = h->generic ? (const void*)hx::hx_sim_kernel : (const void*)hx::hx_sim_kernel_lean;
@@ -398,6 +463,7 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   if ((rc = h->alloc(&h->d_arena, w * h->arena_per_warp)) || (rc = h->alloc(&h->d_chains, w * h->chains_per_warp)) ||
       (rc = h->alloc(&h->d_topk, w * h->topk_per_warp)))
     return bail(rc);
+  if (h->generic && (rc = h->alloc(&h->d_extras, h->n_sims))) return bail(rc);
   h->scratch_bytes = w * (h->arena_per_warp * (int64_t)sizeof(hx::HeapEnt) + h->chains_per_warp +
                           h->topk_per_warp * (int64_t)sizeof(int64_t));
 
@@ -444,6 +510,11 @@ int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* str
   }
   hx_cluster c{};
   c.rmax = h->ck.rmax;
+  c.n_inst = h->ck.n_inst;
+  c.n_tenants = h->n_tenants;
+  c.timeout_mult_fp = h->ck.timeout_mult_fp;
+  c.n_faults = (int32_t)h->faults.size();
+  c.faults = h->faults.data();
   for (int t = 0; t < n_traces; ++t) {
     int rc = validate_trace(&traces[t], t, &c, min_prefill, max_decode);
     if (rc) return rc;
@@ -466,6 +537,7 @@ int hx_sim_run(hx_sim* h, void* stream) {
   pa.stage = h->d_stage;
   pa.cand = h->d_cand;
   pa.retry = h->d_retry;
+  pa.tenant = h->d_tenant;
   pa.n_queries = h->n_q;
   pa.n_traces = h->n_traces;
   pa.rec = h->d_rec;
@@ -500,6 +572,7 @@ int hx_sim_run(hx_sim* h, void* stream) {
   sa.rec_budget = h->d_rec_budget;
   sa.rec_start = h->d_rec_start;
   sa.rec_stride = h->rec_stride;
+  sa.extras = h->d_extras;
 
   hx::BestArgs ba;
   ba.results = h->d_results;
@@ -535,6 +608,28 @@ int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n) {
   if ((int64_t)n > h->n_sims) return fail(HX_ERR_INVALID, "n exceeds the number of simulations");
   HX_CUDA(cudaStreamSynchronize(h->last_stream));
   HX_CUDA(cudaMemcpy(host_out, h->d_results, n * sizeof(hx_result), cudaMemcpyDeviceToHost));
+  return HX_OK;
+}
+
+int hx_sim_extras(hx_sim* h, hx_extra* host_out, size_t n) {
+  if (!h || !host_out) return fail(HX_ERR_INVALID, "NULL argument");
+  if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
+  if ((int64_t)n > h->n_sims) return fail(HX_ERR_INVALID, "n exceeds the number of simulations");
+  HX_CUDA(cudaStreamSynchronize(h->last_stream));
+  if (n == 0) return HX_OK;
+  if (h->d_extras) {
+    HX_CUDA(cudaMemcpy(host_out, h->d_extras, n * sizeof(hx_extra), cudaMemcpyDeviceToHost));
+    return HX_OK;
+  }
+  // the lean kernel serves one tenant without faults: everything is tenant 0
+  std::vector<hx_result> res(n);
+  HX_CUDA(cudaMemcpy(res.data(), h->d_results, n * sizeof(hx_result), cudaMemcpyDeviceToHost));
+  for (size_t i = 0; i < n; ++i) {
+    hx_extra e{};
+    e.slo_met[0] = res[i].slo_met;
+    e.n_done[0] = res[i].n_done;
+    host_out[i] = e;
+  }
   return HX_OK;
 }
 
@@ -798,42 +893,14 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   const int64_t nq = trace->n_queries, nc = trace->n_calls, P = grid->n_points;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
 
-  hx::ClusterK ck{};
-  ck.n_inst = cluster->n_inst;
-  ck.n_types = cluster->n_types;
-  ck.ref_type = cluster->ref_type;
-  ck.rmax = cluster->rmax;
-  ck.slo_mult_fp = cluster->slo_mult_fp;
-  for (int t = 0; t < HX_MAX_TYPES; ++t) {
-    const bool on = t < cluster->n_types;
-    ck.prefill[t] = on ? cluster->prefill_tok_s[t] : 1;
-    ck.decode[t] = on ? cluster->decode_us_tok[t] : 0;
-    ck.slots[t] = on ? cluster->slots[t] : 0;
-    ck.cnt[t] = 0;
-  }
-  for (int st = 0; st < 4; ++st) {
-    ck.ref_prompt[st] = cluster->stage_ref_prompt[st];
-    ck.ref_out[st] = cluster->stage_ref_out[st];
-  }
-  int base = 0;
-  for (int m = 0; m < HX_MAX_INST; ++m) {
-    const bool on = m < cluster->n_inst;
-    const int ty = on ? cluster->inst_type[m] : 0;
-    ck.inst_type[m] = (uint8_t)ty;
-    ck.inst_slots[m] = on ? (uint8_t)cluster->slots[ty] : 0;
-    ck.slot_base[m] = (uint16_t)base;
-    if (on) {
-      base += cluster->slots[ty];
-      ck.cnt[ty]++;
-    }
-  }
-  ck.total_slots = base;
-  ck.smem_per_warp = per_warp_smem(base);
+  hx::ClusterK ck;
+  fill_cluster(cluster, ck);
 
   // layout of the static array: inputs, records, results, then per-warp scratch
   Carve cv;
   const int64_t o_qoff = cv.take<int64_t>(2), o_coff = cv.take<int64_t>(2), o_ctr = cv.take<unsigned long long>(1);
   const int64_t o_arr = cv.take<int64_t>(nq), o_k = cv.take<uint8_t>(nq), o_cb32 = cv.take<int32_t>(nq + 1);
+  const int64_t o_ten = cv.take<uint8_t>(nq);
   const int64_t o_qcall = cv.take<int64_t>(nq + 1);
   const int64_t o_prompt = cv.take<int32_t>(nc), o_out = cv.take<int32_t>(nc), o_oest = cv.take<int32_t>(nc);
   const int64_t o_stage = cv.take<uint8_t>(nc), o_cand = cv.take<uint8_t>(nc), o_retry = cv.take<uint8_t>(nc);
@@ -883,6 +950,7 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
     const void* src;
     int64_t bytes;
   } ups[] = {{o_arr, trace->arrival_us, nq * 8},     {o_k, trace->k, nq},
+             {o_ten, trace->tenant, trace->tenant ? nq : 0},
              {o_cb32, trace->call_base, (nq + 1) * 4}, {o_prompt, trace->prompt, nc * 4},
              {o_out, trace->out, nc * 4},             {o_oest, trace->out_est, nc * 4},
              {o_stage, trace->stage, nc},             {o_cand, trace->cand, nc},
@@ -908,6 +976,7 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   pa.stage = static_cast<const uint8_t*>(at(o_stage));
   pa.cand = static_cast<const uint8_t*>(at(o_cand));
   pa.retry = static_cast<const uint8_t*>(at(o_retry));
+  pa.tenant = trace->tenant ? static_cast<const uint8_t*>(at(o_ten)) : nullptr;
   pa.n_queries = nq;
   pa.n_traces = 1;
   pa.rec = static_cast<hx::CallRec*>(at(o_rec));
@@ -942,6 +1011,7 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   sa.rec_budget = nullptr;
   sa.rec_start = nullptr;
   sa.rec_stride = 0;
+  sa.extras = nullptr;
 
   hx::BestArgs ba;
   ba.results = sa.results;

@@ -39,8 +39,9 @@ struct __align__(16) CallRec {
   int32_t tbar;       // mean of est over the instances
   int32_t next;       // S: unused; G/C: next correction's id, or ~(E's id) at chain end
   int32_t qid;        // query index within the trace
-  uint8_t stage, u, k, fcode;  // stage, corrections done incl. this call, k of the query,
-                               // row of the rest-of-path table: S 0, G/C 1 + u, E 17
+  uint8_t stage, u, k, fcode;  // stage, corrections done incl. this call (E: the query's
+                               // tenant), k of the query, row of the rest-of-path table:
+                               // S 0, G/C 1 + u, E 17
 };
 static_assert(sizeof(CallRec) == 64, "CallRec is one 64-byte unit");
 
@@ -49,6 +50,12 @@ struct __align__(16) HeapEnt {
   long long key;
   int rid;
   int svc;   // service time on the queue's instance
+};
+
+// A fault window of one instance (see hx_fault).
+struct FaultK {
+  int64_t t0, t1, slow;
+  int32_t inst, pad;
 };
 
 // Cluster description passed by value (kernel parameter space).
@@ -62,6 +69,11 @@ struct ClusterK {
   uint8_t inst_type[HX_MAX_INST];
   uint8_t inst_slots[HX_MAX_INST];
   uint16_t slot_base[HX_MAX_INST];
+  // tenants and faults (only the generic simulation kernel handles faults)
+  int32_t n_tenants, n_faults;
+  int64_t tenant_mult[HX_MAX_TENANTS];
+  int64_t timeout_mult_fp;
+  FaultK faults[HX_MAX_FAULTS];
 };
 
 struct PrepArgs {
@@ -76,6 +88,7 @@ struct PrepArgs {
   const uint8_t* stage;
   const uint8_t* cand;
   const uint8_t* retry;
+  const uint8_t* tenant;    // [Q] or NULL
   int64_t n_queries;
   int32_t n_traces;
   CallRec* rec;             // [C]
@@ -111,6 +124,7 @@ struct SimArgs {
   int64_t* rec_budget;
   int64_t* rec_start;
   int64_t rec_stride;
+  hx_extra* extras;         // [n_sims] per-tenant counts and re-issues (generic kernel), or NULL
 };
 
 // Per-warp shared memory of one simulation: per-instance local-queue and
@@ -149,7 +163,9 @@ struct WarpShared {
   int64_t tkmin;                // root of the full top-K heap (written alike by every lane)
   longlong2 dterm[16];          // digest terms waiting to be hashed: (time, id tag)
   int32_t dn, pad1;             // terms waiting (written alike by every lane)
-  uint64_t slot[1];             // [total_slots]
+  int32_t tslo[HX_MAX_TENANTS], tdone[HX_MAX_TENANTS];  // per-tenant counts (generic kernel)
+  int32_t reissued, excl;       // timed-out attempts; the instance a re-issue avoids (-1: none)
+  uint64_t slot[1];             // [total_slots], then with faults one fail flag byte per slot
 };
 
 struct BestCand {

@@ -145,7 +145,9 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
   }
   int64_t longest = 0;
   for (int i = 0; i < k; ++i) longest = chain[i] > longest ? chain[i] : longest;
-  const int64_t t_slo = (c.slo_mult_fp * (l_s + longest + l_e)) / kScale;
+  const int tenant = a.tenant ? a.tenant[g] : 0;
+  const int64_t mult = c.n_tenants > 1 ? c.tenant_mult[tenant] : c.slo_mult_fp;
+  const int64_t t_slo = (mult * (l_s + longest + l_e)) / kScale;
   const int64_t deadline = arr + t_slo;
   const int32_t e_rid = (int32_t)(e - 1 - cbase);
 
@@ -179,7 +181,7 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
       r.fcode = 0;
       r.next = -1;
     } else if (st == HX_STAGE_E) {
-      r.u = 0;
+      r.u = (uint8_t)tenant;
       r.fcode = kFRows - 1;
       r.next = -1;
     } else {
@@ -557,6 +559,12 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       W->events = 0;
       W->tk = 0;
       W->tkmin = 0;
+      for (int t = 0; t < HX_MAX_TENANTS; ++t) {
+        W->tslo[t] = 0;
+        W->tdone[t] = 0;
+      }
+      W->reissued = 0;
+      W->excl = -1;
     }
     __syncwarp();
 
@@ -580,16 +588,46 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     int64_t now = 0;
     int32_t status = HX_OK, npend = 0;
     uint64_t touched = 0;
-    int32_t steps_left = nc + nq + 8;
+    // event bound; re-issued attempts add events while fault windows last
+    const bool faults = kGeneric && c.n_faults > 0;
+    int32_t steps_left = nc + nq + 8 + (faults ? 16 * nc + 4096 : 0);
 
     // Request rid starts on instance m now and runs until now + svc: its key
     // joins the cn sorted keys of m's running calls at sl.
     auto start_call = [&](uint64_t* sl, int m, int cn, int rid, int svc) {
-      const uint64_t nk = ((uint64_t)(now + svc) << 24) | (uint64_t)(uint32_t)rid;
+      int64_t run = svc;
+      bool fail = false;
+      if (faults) {
+        // the first fault window of m that covers now, and the timeout (Sec. 3.3)
+        bool in_window = false, down = false;
+        for (int f = 0; f < c.n_faults; ++f) {
+          const FaultK& F = c.faults[f];
+          if (F.inst == m && now >= F.t0 && now < F.t1) {
+            in_window = true;
+            if (F.slow == 0) down = true;
+            else run = (run * F.slow + kScale - 1) / kScale;
+            break;
+          }
+        }
+        if (in_window && c.timeout_mult_fp > 0) {
+          const int64_t timeout = ((int64_t)rec[rid].est[c.inst_type[m]] * c.timeout_mult_fp) / kScale;
+          if (down || run > timeout) {
+            fail = true;
+            run = timeout;
+          }
+        }
+      }
+      const uint64_t nk = ((uint64_t)(now + run) << 24) | (uint64_t)(uint32_t)rid;
       const uint64_t cur = lane < cn ? sl[lane] : kKeyInf;
+      uint8_t* const fl = faults ? reinterpret_cast<uint8_t*>(W->slot + c.total_slots) + (sl - W->slot) : nullptr;
+      const uint8_t fcur = (faults && lane < cn) ? fl[lane] : 0;
       const int pos = __popc(__ballot_sync(kFull, cur < nk));
       if (lane >= pos && lane < cn) sl[lane + 1] = cur;
       if (lane == pos) sl[pos] = nk;
+      if (faults) {
+        if (lane >= pos && lane < cn) fl[lane + 1] = fcur;
+        if (lane == pos) fl[pos] = fail ? 1 : 0;
+      }
       digest_push(W, now, call_tag(rid, m), lane);
       if (kGeneric && lane == 0) {
         const int recj = W->recj;
@@ -634,8 +672,12 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         // remove it: the remaining keys move down one slot
         const uint64_t nxt = lane + 1 < cn ? sl[lane + 1] : kKeyInf;
         const uint64_t head = cn > 1 ? sl[1] : kKeyInf;
+        uint8_t* const fl = faults ? reinterpret_cast<uint8_t*>(W->slot + c.total_slots) + (sl - W->slot) : nullptr;
+        const bool failed = faults && fl[0] != 0;
+        const uint8_t fnxt = (faults && lane + 1 < cn) ? fl[lane + 1] : 0;
         __syncwarp();
         if (lane < cn) sl[lane] = nxt;
+        if (faults && lane < cn) fl[lane] = fnxt;
         if (lane == 0) W->cnt[m] = cn - 1;
         set_key(m, head);
         if (lane == (m & 31)) {
@@ -648,13 +690,25 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         if (hs_m > 0) touched |= 1ull << m;
         const int stg = tail.w & 0xff;
         const int32_t qid = tail.z;
-        if (stg == HX_STAGE_S) {
+        if (faults && failed) {
+          // the attempt timed out: the request goes out again, avoiding m
+          if (lane == 0) W->reissued++;
+          W->excl = c.n_inst > 1 ? m : -1;
+          rel_first = rid;
+          rel_count = 1;
+        } else if (stg == HX_STAGE_S) {
           const int k = (tail.w >> 16) & 0xff;
           if (lane == 0) W->chains[qid] = (uint8_t)k;
           rel_first = rid + 1;
           rel_count = k;
         } else if (stg == HX_STAGE_E) {
-          finish_query(W, qid, now, r->arrival, r->deadline, lane);
+          const int64_t dl = r->deadline;
+          if (kGeneric && lane == 0) {
+            const int ten = (tail.w >> 8) & 0xff;
+            W->tdone[ten]++;
+            W->tslo[ten] += now <= dl ? 1 : 0;
+          }
+          finish_query(W, qid, now, r->arrival, dl, lane);
         } else {
           const int32_t nx = tail.y;
           if (nx >= 0) {
@@ -701,17 +755,25 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           else if (dirty1) { orew1 = orew; dirty1 = false; }
         }
         int m;
+        // a re-issued request avoids the instance it timed out on
+        const int excl = kGeneric ? W->excl : -1;
         if (kGeneric && W->dpol == HX_DISPATCH_RR) {
           m = W->rr;
+          if (m == excl) m = (m + 1 == N) ? 0 : m + 1;
           __syncwarp();
           if (lane == 0) W->rr = (m + 1 == N) ? 0 : m + 1;
         } else {
           const int32_t A = W->A;
-          const int64_t s0 = orew0 - (int64_t)A * e0;
-          const int64_t s1 = orew1 - (int64_t)A * e1;
+          int64_t s0 = orew0 - (int64_t)A * e0;
+          int64_t s1 = orew1 - (int64_t)A * e1;
+          if (kGeneric && excl >= 0) {
+            if (m0 == excl) s0 = INT64_MIN;
+            if (m1 == excl) s1 = INT64_MIN;
+          }
           const bool take1 = s1 > s0;
           m = warp_argmax_s64(take1 ? s1 : s0, take1 ? m1 : m0);
         }
+        if (kGeneric) W->excl = -1;
         // the winner's costs, from the lane that owns it
         const int64_t est_m = __shfl_sync(kFull, m < 32 ? e0 : e1, m & 31);
         const int svc_m = __shfl_sync(kFull, m < 32 ? v0 : v1, m & 31);
@@ -816,7 +878,8 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       hx_result res;
       res.p95_us = st == HX_OK ? (nq > 0 ? W->topk[0] : 0) : -1;
       res.makespan_us = W->makespan;
-      res.events = (W->nc + nq + 8 - steps_left) - W->qa;
+      const int32_t steps0 = W->nc + nq + 8 + (kGeneric && c.n_faults > 0 ? 16 * W->nc + 4096 : 0);
+      res.events = (steps0 - steps_left) - W->qa - (kGeneric ? W->reissued : 0);
       res.digest = W->digest;
       res.slo_met = W->slo_met;
       res.n_done = n_done;
@@ -824,6 +887,16 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       const long long dc = (clock64() - W->clk0) >> 10;
       res.cycles_k = dc < INT32_MAX ? (int32_t)dc : INT32_MAX;
       a.results[W->sim] = res;
+      if (kGeneric && a.extras) {
+        hx_extra ex;
+        for (int t = 0; t < HX_MAX_TENANTS; ++t) {
+          ex.slo_met[t] = W->tslo[t];
+          ex.n_done[t] = W->tdone[t];
+        }
+        ex.reissued = W->reissued;
+        ex.pad = 0;
+        a.extras[W->sim] = ex;
+      }
     }
     __syncwarp();
   }

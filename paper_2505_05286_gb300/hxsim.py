@@ -28,6 +28,7 @@ OBJ_P95, OBJ_P95_SLO95 = 0, 1
 RESULT_DTYPE = np.dtype([("p95_us", "<i8"), ("makespan_us", "<i8"), ("events", "<i8"),
                          ("digest", "<u8"), ("slo_met", "<i4"), ("n_done", "<i4"),
                          ("status", "<i4"), ("cycles_k", "<i4")])
+EXTRA_DTYPE = np.dtype([("slo_met", "<i4", (4,)), ("n_done", "<i4", (4,)), ("reissued", "<i4"), ("pad", "<i4")])
 
 
 class HxError(RuntimeError):
@@ -40,7 +41,13 @@ class hx_trace(ctypes.Structure):
     _fields_ = [("n_queries", ctypes.c_int32), ("n_calls", ctypes.c_int32),
                 ("arrival_us", ctypes.c_void_p), ("k", ctypes.c_void_p), ("call_base", ctypes.c_void_p),
                 ("prompt", ctypes.c_void_p), ("out", ctypes.c_void_p), ("out_est", ctypes.c_void_p),
-                ("stage", ctypes.c_void_p), ("cand", ctypes.c_void_p), ("retry", ctypes.c_void_p)]
+                ("stage", ctypes.c_void_p), ("cand", ctypes.c_void_p), ("retry", ctypes.c_void_p),
+                ("tenant", ctypes.c_void_p)]
+
+
+class hx_fault(ctypes.Structure):
+    _fields_ = [("inst", ctypes.c_int32), ("pad", ctypes.c_int32), ("t0_us", ctypes.c_int64),
+                ("t1_us", ctypes.c_int64), ("slow_fp", ctypes.c_int64)]
 
 
 class hx_cluster(ctypes.Structure):
@@ -48,7 +55,9 @@ class hx_cluster(ctypes.Structure):
                 ("decode_us_tok", ctypes.c_void_p), ("slots", ctypes.c_void_p), ("n_inst", ctypes.c_int32),
                 ("inst_type", ctypes.c_void_p), ("ref_type", ctypes.c_int32), ("slo_mult_fp", ctypes.c_int64),
                 ("rmax", ctypes.c_int32), ("stage_ref_prompt", ctypes.c_void_p),
-                ("stage_ref_out", ctypes.c_void_p)]
+                ("stage_ref_out", ctypes.c_void_p), ("n_tenants", ctypes.c_int32), ("n_faults", ctypes.c_int32),
+                ("tenant_slo_mult_fp", ctypes.c_void_p), ("timeout_mult_fp", ctypes.c_int64),
+                ("faults", ctypes.c_void_p)]
 
 
 class hx_grid(ctypes.Structure):
@@ -106,7 +115,7 @@ def load(path: Optional[str] = None):
                        ("hx_sim_info", [vp, vp]), ("hx_sim_destroy", [vp]),
                        ("hx_sim_run_static", [vp, vp, vp, i32, vp, vp, vp]),
                        ("hx_selftest_div", [vp, vp, vp, vp, sz]),
-                       ("hx_sim_point_sums", [vp, vp, vp, vp, sz]),
+                       ("hx_sim_point_sums", [vp, vp, vp, vp, sz]), ("hx_sim_extras", [vp, vp, sz]),
                        ("hx_best_of_sums", [vp, vp, vp, i32, ctypes.c_int64, i32, vp])]:
         fn = getattr(lib, name)
         fn.restype = ctypes.c_int
@@ -148,6 +157,8 @@ class _Traces:
             cols = [_c(t.arrival_us, np.int64), _c(t.k, np.uint8), _c(t.call_base, np.int32),
                     _c(t.prompt, np.int32), _c(t.out, np.int32), _c(t.out_est, np.int32),
                     _c(t.stage, np.uint8), _c(t.cand, np.uint8), _c(t.retry, np.uint8)]
+            ten = getattr(t, "tenant", None)
+            cols.append(None if ten is None else _c(ten, np.uint8))
             self.keep.append(cols)
             self.arr[i] = hx_trace(int(cols[0].shape[0]), int(cols[3].shape[0]), *[_p(x) for x in cols])
 
@@ -176,8 +187,19 @@ def best_of_sums(sum_p95, sum_slo_met, n_failed, n_queries_total: int, objective
 def _cluster_struct(c):
     cols = [_c(c.prefill_tok_s, np.int32), _c(c.decode_us_tok, np.int32), _c(c.slots, np.int32),
             _c(c.inst_type, np.uint8), _c(c.stage_ref_prompt, np.int32), _c(c.stage_ref_out, np.int32)]
+    tm = getattr(c, "tenant_slo_mult_fp", None)
+    tm = None if tm is None else _c(tm, np.int64)
+    fl = getattr(c, "faults", None)
+    n_f = 0 if fl is None else len(fl)
+    faults = (hx_fault * max(n_f, 1))()
+    for j in range(n_f):
+        f = fl[j]
+        faults[j] = hx_fault(int(f["inst"]), 0, int(f["t0_us"]), int(f["t1_us"]), int(f["slow_fp"]))
+    cols += [tm, faults]
     st = hx_cluster(int(cols[0].shape[0]), _p(cols[0]), _p(cols[1]), _p(cols[2]), int(cols[3].shape[0]),
-                    _p(cols[3]), int(c.ref_type), int(c.slo_mult_fp), int(c.rmax), _p(cols[4]), _p(cols[5]))
+                    _p(cols[3]), int(c.ref_type), int(c.slo_mult_fp), int(c.rmax), _p(cols[4]), _p(cols[5]),
+                    0 if tm is None else int(tm.shape[0]), n_f, _p(tm), int(getattr(c, "timeout_mult_fp", 0)),
+                    ctypes.cast(faults, ctypes.c_void_p) if n_f else None)
     return st, cols
 
 
@@ -213,15 +235,8 @@ class Sim:
         self.n_calls = [int(t.prompt.shape[0]) for t in traces]
         self.n_queries = [int(t.arrival_us.shape[0]) for t in traces]
         tr = _Traces(traces)
-        c = cluster
-        ccols = [_c(c.prefill_tok_s, np.int32), _c(c.decode_us_tok, np.int32), _c(c.slots, np.int32),
-                 _c(c.inst_type, np.uint8), _c(c.stage_ref_prompt, np.int32), _c(c.stage_ref_out, np.int32)]
-        hc = hx_cluster(int(ccols[0].shape[0]), _p(ccols[0]), _p(ccols[1]), _p(ccols[2]), int(ccols[3].shape[0]),
-                        _p(ccols[3]), int(c.ref_type), int(c.slo_mult_fp), int(c.rmax), _p(ccols[4]), _p(ccols[5]))
-        g = grid
-        gcols = [_c(g.alpha_fp, np.int64), _c(g.gamma_fp, np.int64), _c(g.rho, np.int32), _c(g.beta_us2, np.int64),
-                 _c(g.local_policy, np.uint8), _c(g.dispatch_policy, np.uint8)]
-        hg = hx_grid(self.n_points, *[_p(x) for x in gcols])
+        hc, keep_c = _cluster_struct(cluster)
+        hg, keep_g = _grid_struct(grid)
         self.record_sims = [int(s) for s in record_sims]
         rs = _c(self.record_sims if self.record_sims else [0], np.int32)
         opt = hx_options(len(self.record_sims), _p(rs), int(max_resident_warps), int(bool(timing)),
@@ -245,6 +260,12 @@ class Sim:
     def results(self) -> np.ndarray:
         out = np.zeros(self.n_sims, RESULT_DTYPE)
         _check(self.lib, self.lib.hx_sim_results(self.h, _p(out), self.n_sims))
+        return out
+
+    def extras(self) -> np.ndarray:
+        """Per-tenant SLO hits and completed queries, and re-issued attempts, one row per sim."""
+        out = np.zeros(self.n_sims, EXTRA_DTYPE)
+        _check(self.lib, self.lib.hx_sim_extras(self.h, _p(out), self.n_sims))
         return out
 
     def best(self, objective: int = OBJ_P95):

@@ -18,7 +18,10 @@ order.
 The five workload recipes (`CONFIGS`) stand in for the paper's BIRD / Spider
 derived traces (Sec. 5.1), which are not available: Poisson or two-state MMPP
 query arrivals, per-stage token-length distributions (uniform or clipped
-lognormal), candidate counts k, error probability p and retry limit R.
+lognormal), candidate counts k, error probability p and retry limit R.  The
+`EXTRA` recipes add Sec. 5's other settings: ~20 calls per query, a noisy
+output-length predictor, two tenants with different SLOs, competing
+single-shot requests, and instances that slow down or stop for a while.
 """
 from __future__ import annotations
 
@@ -44,6 +47,10 @@ OBJ_P95 = 0        # argmin P95 (Sec. 4.3)
 OBJ_P95_SLO95 = 1  # argmin P95 among points with >= 95% SLO attainment
 
 SCALE = 1_000_000  # fixed-point scale of alpha, gamma and the SLO multiplier
+
+# A fault window: attempts that start on `inst` in [t0_us, t1_us) run
+# slow_fp / SCALE times longer; slow_fp = 0 stops them (they time out).
+FAULT_DTYPE = np.dtype([("inst", "<i4"), ("pad", "<i4"), ("t0_us", "<i8"), ("t1_us", "<i8"), ("slow_fp", "<i8")])
 
 _M64 = (1 << 64) - 1
 _GOLD = 0x9E3779B97F4A7C15
@@ -74,6 +81,7 @@ class Trace:
     stage: np.ndarray       # uint8 [nc]
     cand: np.ndarray        # uint8 [nc]
     retry: np.ndarray       # uint8 [nc]
+    tenant: Optional[np.ndarray] = None  # uint8 [nq] tenant of each query (None: all tenant 0)
 
     @property
     def n_queries(self) -> int:
@@ -97,6 +105,13 @@ class Cluster:
     rmax: int                   # configured retry bound R of the workflow
     stage_ref_prompt: np.ndarray  # int32 [4] reference prompt length per stage
     stage_ref_out: np.ndarray     # int32 [4] reference output length per stage
+    tenant_slo_mult_fp: Optional[np.ndarray] = None  # int64 [n_tenants] per-tenant SLO multipliers
+    timeout_mult_fp: int = 0      # attempt timeout as a multiple of its estimate (0: none)
+    faults: Optional[np.ndarray] = None  # FAULT_DTYPE [n_faults] instance slow-down / outage windows
+
+    @property
+    def n_tenants(self) -> int:
+        return 1 if self.tenant_slo_mult_fp is None else int(len(self.tenant_slo_mult_fp))
 
     @property
     def n_types(self) -> int:
@@ -178,6 +193,7 @@ def stream_uniform(key: int, n: int, start: int = 0) -> np.ndarray:
 
 
 _STREAM_ARRIVAL, _STREAM_DWELL, _STREAM_K, _STREAM_ERR, _STREAM_PROMPT, _STREAM_OUT, _STREAM_EST = range(1, 8)
+_STREAM_TENANT, _STREAM_SINGLE = 8, 9
 
 
 # ----------------------------------------------------------------------------
@@ -219,6 +235,12 @@ class Recipe:
     objective: int
     trace_seeds: Optional[Sequence[int]] = None
     est_noise_sigma: float = 0.0  # lognormal noise of the believed output length (0: the stage mean)
+    tenant_slo_mult_fp: Optional[Sequence[int]] = None  # per-tenant SLO multipliers (None: one tenant)
+    tenant_share: Optional[Sequence[float]] = None      # tenant probabilities of the workflow queries
+    single_frac: float = 0.0      # single-shot requests added, as a fraction of the workflow's calls
+    single_tenant: int = 0        # tenant of the single-shot requests
+    timeout_mult: float = 0.0     # attempt timeout as a multiple of its estimate (0: none)
+    faults: Optional[Sequence[Sequence[float]]] = None  # (instance, t0 s, t1 s, slow-down; 0 = stopped)
 
 
 def _u(a, b):
@@ -276,7 +298,20 @@ CONFIGS: List[Recipe] = [
 #  - "paper-shaped": ~20 calls per query (k = 8 candidates, error probability
 #    0.55, up to 10 refinement rounds) at 1 query/s on a 2A + 2B cluster;
 #  - "noisy-estimate": recipe 1 with the output-length predictor replaced by
-#    the true length times lognormal(0, 0.5) noise.
+#    the true length times lognormal(0, 0.5) noise;
+#  - "two-tenant": recipe 1 with two tenants, SLO 2x and 4x, half the
+#    queries each (the multi-tenant evaluation);
+#  - "competing-25" / "competing-50": recipe 1 plus single-shot requests
+#    numbering 25% / 50% of the workflow's calls, with generation-stage token
+#    lengths and their own tenant and SLO (5x);
+#  - "faulty": recipe 1 with a 3x-estimate timeout, instance 0 (type A)
+#    stopped for 60 s, instance 4 (type B) 3x slower for 120 s and instance
+#    6 (type C) stopped for 30 s (timeout and re-issue, Sec. 3.3).
+_SMALL = dict(n_traces=8, n_queries=2000, arrival="poisson", rate_qps=[4.0], mmpp_dwell_s=0.0, k_range=[4, 4],
+              p_err=0.3, rmax=2, prompt=_UNIF_PROMPT, out=_UNIF_OUT, out_est=_UNIF_OUT_EST,
+              ref_prompt=_UNIF_REF_PROMPT, types=[TYPE_A, TYPE_B, TYPE_C], inst_counts=[4, 2, 2], ref_type=0,
+              slo_mult_fp=3 * SCALE, alpha_n=8, gamma_fp=_GAMMA8, rho=None, beta_mult=[(1, 1)], c_ref_us=300_000,
+              objective=OBJ_P95)
 EXTRA: dict = {
     "paper-shaped": Recipe("paper-shaped-8x400q-4inst-16pt", 8, 400, "poisson", [1.0], 0.0, [8, 8], 0.55, 10,
                            _UNIF_PROMPT, _UNIF_OUT, _UNIF_OUT_EST, _UNIF_REF_PROMPT,
@@ -286,7 +321,18 @@ EXTRA: dict = {
                              _UNIF_PROMPT, _UNIF_OUT, _UNIF_OUT_EST, _UNIF_REF_PROMPT,
                              [TYPE_A, TYPE_B, TYPE_C], [4, 2, 2], 0, 3 * SCALE,
                              8, _GAMMA8, None, [(1, 1)], 300_000, OBJ_P95, est_noise_sigma=0.5),
+    "two-tenant": Recipe("two-tenant-8x2000q-8inst-64pt", **_SMALL, tenant_slo_mult_fp=[2 * SCALE, 4 * SCALE],
+                         tenant_share=[0.5, 0.5]),
+    "competing-25": Recipe("competing25-8x2000q-8inst-64pt", **_SMALL, tenant_slo_mult_fp=[3 * SCALE, 5 * SCALE],
+                           single_frac=0.25, single_tenant=1),
+    "competing-50": Recipe("competing50-8x2000q-8inst-64pt", **_SMALL, tenant_slo_mult_fp=[3 * SCALE, 5 * SCALE],
+                           single_frac=0.5, single_tenant=1),
+    "faulty": Recipe("faulty-8x2000q-8inst-64pt", **_SMALL, timeout_mult=3.0,
+                     faults=[(0, 100.0, 160.0, 0.0), (4, 200.0, 320.0, 3.0), (6, 300.0, 330.0, 0.0)]),
 }
+# Random-stream ids of the extra recipes (fixed, so adding one changes no other trace).
+EXTRA_ID = {"noisy-estimate": 16, "paper-shaped": 17, "two-tenant": 18, "competing-25": 19, "competing-50": 20,
+            "faulty": 21}
 
 
 # ----------------------------------------------------------------------------
@@ -426,17 +472,69 @@ def make_trace(recipe: Recipe, cfg_id: int, seed: int, n_queries: Optional[int] 
         z = np.sqrt(-2.0 * np.log(1.0 - ue[:, 0])) * np.cos(2.0 * np.pi * ue[:, 1])
         est = np.floor(out.astype(np.float64) * np.exp(recipe.est_noise_sigma * z) + 0.5)
         out_est = np.clip(est, 0, 1 << 20).astype(np.int32)
-    return Trace(arrival.astype(np.int64), k.astype(np.uint8), call_base.astype(np.int32),
-                 prompt, out, out_est.astype(np.int32), stage, cand, retry)
+    tr = Trace(arrival.astype(np.int64), k.astype(np.uint8), call_base.astype(np.int32),
+               prompt, out, out_est.astype(np.int32), stage, cand, retry)
+    if recipe.tenant_share is not None:
+        ut = stream_uniform(stream_key(key, _STREAM_TENANT), nq)
+        cum = np.cumsum(np.asarray(recipe.tenant_share, np.float64))
+        tr.tenant = np.minimum(np.searchsorted(cum / cum[-1], ut, side="right"), len(cum) - 1).astype(np.uint8)
+    if recipe.single_frac > 0:
+        tr = _add_single_shots(tr, recipe, key)
+    return tr
+
+
+def _add_single_shots(tr: Trace, recipe: Recipe, key: int) -> Trace:
+    """Merge independent single-shot requests (a query of one evaluation-stage
+    call, k = 0) into a trace: single_frac x its calls of them, Poisson over
+    the trace's span, generation-stage token lengths, tenant single_tenant."""
+    ns = int(np.floor(recipe.single_frac * tr.n_calls + 0.5))
+    if ns == 0 or tr.n_queries == 0:
+        return tr
+    ks = stream_key(key, _STREAM_SINGLE)
+    span_s = max(int(tr.arrival_us[-1]), 1) / 1e6
+    arr = _poisson_arrivals(ks, ns, ns / span_s)
+    gen = np.full(ns, STAGE_G, np.uint8)
+    s_prompt = _draw_tokens(stream_key(ks, _STREAM_PROMPT), gen, recipe.prompt)
+    s_out = _draw_tokens(stream_key(ks, _STREAM_OUT), gen, recipe.out)
+    s_est = np.full(ns, recipe.out_est[STAGE_G], np.int32)
+    if recipe.est_noise_sigma > 0:
+        ue = stream_uniform(stream_key(ks, _STREAM_EST), 2 * ns).reshape(ns, 2)
+        z = np.sqrt(-2.0 * np.log(1.0 - ue[:, 0])) * np.cos(2.0 * np.pi * ue[:, 1])
+        s_est = np.clip(np.floor(s_out * np.exp(recipe.est_noise_sigma * z) + 0.5), 0, 1 << 20).astype(np.int32)
+    nq0, nc0 = tr.n_queries, tr.n_calls
+    # by arrival, workflow queries first at equal times
+    arr_all = np.concatenate([tr.arrival_us, arr])
+    single = np.concatenate([np.zeros(nq0, np.int64), np.ones(ns, np.int64)])
+    order = np.lexsort((np.arange(nq0 + ns), single, arr_all))
+    cnt = np.concatenate([np.diff(tr.call_base).astype(np.int64), np.ones(ns, np.int64)])[order]
+    call_base = np.zeros(nq0 + ns + 1, np.int64)
+    call_base[1:] = np.cumsum(cnt)
+    src = np.concatenate([tr.call_base[:-1].astype(np.int64), nc0 + np.arange(ns, dtype=np.int64)])[order]
+    idx = np.repeat(src - call_base[:-1], cnt) + np.arange(int(call_base[-1]), dtype=np.int64)
+    cat = lambda base, extra: np.concatenate([base, extra])[idx]
+    z8 = np.zeros(ns, np.uint8)
+    ten0 = tr.tenant if tr.tenant is not None else np.zeros(nq0, np.uint8)
+    return Trace(arr_all[order].astype(np.int64), np.concatenate([tr.k, z8])[order].astype(np.uint8),
+                 call_base.astype(np.int32), cat(tr.prompt, s_prompt).astype(np.int32),
+                 cat(tr.out, s_out).astype(np.int32), cat(tr.out_est, s_est).astype(np.int32),
+                 cat(tr.stage, np.full(ns, STAGE_E, np.uint8)), cat(tr.cand, z8), cat(tr.retry, z8),
+                 np.concatenate([ten0, np.full(ns, recipe.single_tenant, np.uint8)])[order].astype(np.uint8))
 
 
 def make_cluster(recipe: Recipe) -> Cluster:
     t = np.asarray(recipe.types, dtype=np.int64)
     inst = np.repeat(np.arange(len(recipe.types)), recipe.inst_counts).astype(np.uint8)
+    faults = None
+    if recipe.faults:
+        faults = np.zeros(len(recipe.faults), FAULT_DTYPE)
+        for j, (m, t0, t1, slow) in enumerate(recipe.faults):
+            faults[j] = (int(m), 0, int(round(t0 * 1e6)), int(round(t1 * 1e6)), int(round(slow * SCALE)))
+    tmult = None if recipe.tenant_slo_mult_fp is None else np.asarray(recipe.tenant_slo_mult_fp, np.int64)
     return Cluster(t[:, 0].astype(np.int32), t[:, 1].astype(np.int32), t[:, 2].astype(np.int32), inst,
                    int(recipe.ref_type), int(recipe.slo_mult_fp), int(recipe.rmax),
                    np.asarray(recipe.ref_prompt, dtype=np.int32),
-                   np.asarray(recipe.out_est, dtype=np.int32))
+                   np.asarray(recipe.out_est, dtype=np.int32), tmult,
+                   int(round(recipe.timeout_mult * SCALE)), faults)
 
 
 def make_grid(recipe: Recipe, local_policy: int = POLICY_PQ, dispatch_policy: int = DISPATCH_WB) -> Grid:
@@ -460,7 +558,7 @@ def make_workload(cfg_id, n_traces: Optional[int] = None, n_queries: Optional[in
     optionally with fewer traces or queries."""
     r = CONFIGS[cfg_id] if isinstance(cfg_id, int) else EXTRA[cfg_id]
     if not isinstance(cfg_id, int):
-        cfg_id = 16 + sorted(EXTRA).index(cfg_id)
+        cfg_id = EXTRA_ID[cfg_id]
     nt = r.n_traces if n_traces is None else int(n_traces)
     traces = [make_trace(r, cfg_id, first_trace + j, n_queries) for j in range(nt)]
     name = r.name if (n_traces is None and n_queries is None) else (

@@ -16,10 +16,17 @@ def load_golden(name):
 
 
 def cluster_from(d, slo_mult_fp=None):
+    faults = None
+    if d.get("faults"):
+        faults = np.zeros(len(d["faults"]), W.FAULT_DTYPE)
+        for j, (m, t0, t1, slow) in enumerate(d["faults"]):
+            faults[j] = (m, 0, t0, t1, slow)
+    tm = d.get("tenant_slo_mult_fp")
     return W.Cluster(np.array(d["prefill_tok_s"], np.int32), np.array(d["decode_us_tok"], np.int32),
                      np.array(d["slots"], np.int32), np.array(d["inst_type"], np.uint8), int(d["ref_type"]),
                      int(d["slo_mult_fp"] if slo_mult_fp is None else slo_mult_fp), int(d["rmax"]),
-                     np.array(d["stage_ref_prompt"], np.int32), np.array(d["stage_ref_out"], np.int32))
+                     np.array(d["stage_ref_prompt"], np.int32), np.array(d["stage_ref_out"], np.int32),
+                     None if tm is None else np.array(tm, np.int64), int(d.get("timeout_mult_fp", 0)), faults)
 
 
 def trace_from(d):
@@ -36,10 +43,13 @@ def trace_from(d):
             cols["out"].append(c[4])
             cols["out_est"].append(c[5])
         base.append(base[-1] + len(q["calls"]))
+    tenant = None
+    if any("tenant" in q for q in d["queries"]):
+        tenant = np.array([q.get("tenant", 0) for q in d["queries"]], np.uint8)
     return W.Trace(np.array(arrival, np.int64), np.array(k, np.uint8), np.array(base, np.int32),
                    np.array(cols["prompt"], np.int32), np.array(cols["out"], np.int32),
                    np.array(cols["out_est"], np.int32), np.array(cols["stage"], np.uint8),
-                   np.array(cols["cand"], np.uint8), np.array(cols["retry"], np.uint8))
+                   np.array(cols["cand"], np.uint8), np.array(cols["retry"], np.uint8), tenant)
 
 
 def grid_from_points(points):

@@ -35,9 +35,12 @@ _PROBE = r"""
 #define F(T, f) printf(#T "." #f " %zu %zu\n", offsetof(T, f), sizeof(((T*)0)->f));
 #define S(T) printf(#T " %zu\n", sizeof(T));
 int main(void) {
-  S(hx_trace) F(hx_trace, n_queries) F(hx_trace, arrival_us) F(hx_trace, retry)
+  S(hx_trace) F(hx_trace, n_queries) F(hx_trace, arrival_us) F(hx_trace, retry) F(hx_trace, tenant)
   S(hx_cluster) F(hx_cluster, n_inst) F(hx_cluster, inst_type) F(hx_cluster, slo_mult_fp) F(hx_cluster, rmax)
-  F(hx_cluster, stage_ref_out)
+  F(hx_cluster, stage_ref_out) F(hx_cluster, n_faults) F(hx_cluster, tenant_slo_mult_fp)
+  F(hx_cluster, timeout_mult_fp) F(hx_cluster, faults)
+  S(hx_fault) F(hx_fault, t0_us) F(hx_fault, slow_fp)
+  S(hx_extra) F(hx_extra, n_done) F(hx_extra, reissued)
   S(hx_grid) F(hx_grid, alpha_fp) F(hx_grid, dispatch_policy)
   S(hx_options) F(hx_options, record_sims) F(hx_options, timing) F(hx_options, force_generic)
   S(hx_result) F(hx_result, digest) F(hx_result, status) F(hx_result, cycles_k)
@@ -58,30 +61,30 @@ def test_struct_layout_matches_binding(tmp_path):
         parts = line.split()
         got[parts[0]] = tuple(int(x) for x in parts[1:])
     structs = {"hx_trace": H.hx_trace, "hx_cluster": H.hx_cluster, "hx_grid": H.hx_grid,
-               "hx_options": H.hx_options, "hx_best": H.hx_best, "hx_info": H.hx_info}
+               "hx_options": H.hx_options, "hx_best": H.hx_best, "hx_info": H.hx_info, "hx_fault": H.hx_fault}
     for key, val in got.items():
         if "." in key:
             sname, field = key.split(".")
             if sname == "hx_result":
                 assert H.RESULT_DTYPE.fields[field][1] == val[0]
                 continue
+            if sname == "hx_extra":
+                assert H.EXTRA_DTYPE.fields[field][1] == val[0]
+                continue
             ct = structs[sname]
             assert getattr(ct, field).offset == val[0], key
             assert getattr(ct, field).size == val[1], key
         elif key == "hx_result":
             assert H.RESULT_DTYPE.itemsize == val[0]
+        elif key == "hx_extra":
+            assert H.EXTRA_DTYPE.itemsize == val[0]
         else:
             assert ctypes.sizeof(structs[key]) == val[0], key
 
 
 def _create(lib, traces, cluster, grid):
     t = H._Traces(traces)
-    c = cluster
-    cc = [np.ascontiguousarray(x) for x in (c.prefill_tok_s.astype(np.int32), c.decode_us_tok.astype(np.int32),
-                                            c.slots.astype(np.int32), c.inst_type.astype(np.uint8),
-                                            c.stage_ref_prompt.astype(np.int32), c.stage_ref_out.astype(np.int32))]
-    hc = H.hx_cluster(len(cc[0]), H._p(cc[0]), H._p(cc[1]), H._p(cc[2]), len(cc[3]), H._p(cc[3]), c.ref_type,
-                      c.slo_mult_fp, c.rmax, H._p(cc[4]), H._p(cc[5]))
+    hc, keep = H._cluster_struct(cluster)
     g = grid
     gc = [np.ascontiguousarray(g.alpha_fp, np.int64), np.ascontiguousarray(g.gamma_fp, np.int64),
           np.ascontiguousarray(g.rho, np.int32), np.ascontiguousarray(g.beta_us2, np.int64),
@@ -127,6 +130,25 @@ def test_rejects_malformed_inputs_without_device_work(lib):
     t5 = _copy_trace(tr)
     t5.arrival_us[:] += 1 << 40
     cases.append(("horizon", [t5], wl.cluster, wl.grid, "horizon"))
+    t6 = _copy_trace(tr)
+    t6.tenant = np.full(tr.n_queries, 2, np.uint8)
+    c6 = W.Cluster(c.prefill_tok_s, c.decode_us_tok, c.slots, c.inst_type, c.ref_type, c.slo_mult_fp, c.rmax,
+                   c.stage_ref_prompt, c.stage_ref_out, np.array([W.SCALE, 2 * W.SCALE], np.int64))
+    cases.append(("tenant 2 of 2", [t6], c6, wl.grid, "tenant out of range"))
+    t7 = _copy_trace(tr)
+    t7.k[0] = 0
+    cases.append(("k = 0 with a whole workflow", [t7], wl.cluster, wl.grid, "single E call"))
+
+    def faulty(faults, timeout):
+        f = np.zeros(len(faults), W.FAULT_DTYPE)
+        for j, x in enumerate(faults):
+            f[j] = (x[0], 0, x[1], x[2], x[3])
+        return W.Cluster(c.prefill_tok_s, c.decode_us_tok, c.slots, c.inst_type, c.ref_type, c.slo_mult_fp, c.rmax,
+                         c.stage_ref_prompt, c.stage_ref_out, None, timeout, f)
+    cases.append(("stopped without timeout", [tr], faulty([(0, 0, 100, 0)], 0), wl.grid, "needs a timeout"))
+    cases.append(("fault instance", [tr], faulty([(4, 0, 100, W.SCALE)], 0), wl.grid, "fault instance"))
+    cases.append(("fault window", [tr], faulty([(0, 100, 50, W.SCALE)], 0), wl.grid, "fault window"))
+    cases.append(("timeout < 1", [tr], faulty([(0, 0, 100, 0)], W.SCALE // 2), wl.grid, "timeout_mult_fp"))
     for name, trs, cl, gr, msg in cases:
         rc, err, h = _create(lib, trs, cl, gr)
         assert rc == H.HX_ERR_INVALID, name

@@ -81,6 +81,10 @@ def test_hand_case(name):
         assert lg["budget"].tolist() == exp["budget"]
     assert int(r["p95_us"]) == exp["p95_us"] and int(r["slo_met"]) == exp["slo_met"]
     assert int(r["makespan_us"]) == exp["makespan_us"]
+    if "tenant_slo_met" in exp:
+        e = sim.extras()[0]
+        assert e["slo_met"].tolist() == exp["tenant_slo_met"] and e["n_done"].tolist() == exp["tenant_done"]
+        assert int(e["reissued"]) == exp["reissued"]
     sim.close()
 
 
@@ -326,3 +330,48 @@ def test_lean_and_generic_kernels_agree():
     assert_same(lean.results()[list(range(0, wl.n_sims, 37)) + [wl.n_sims - 1]], o, "lean vs oracle")
     lean.close()
     full.close()
+
+
+def assert_extras(g, o, what=""):
+    for f in ("slo_met", "n_done", "reissued"):
+        bad = np.nonzero((g[f] != o[f]).reshape(len(g), -1).any(axis=1))[0]
+        assert bad.size == 0, f"{what} extra field {f} differs at {bad[:8].tolist()}"
+
+
+@pytest.mark.parametrize("name,nt,nq", [("two-tenant", 2, 400), ("competing-25", 2, 300), ("competing-50", 1, 300),
+                                        ("faulty", 1, 1400)])
+def test_tenants_single_shots_faults_every_sim(name, nt, nq):
+    """Two tenants with their own SLOs, competing single-shot requests, and
+    instances that slow down or stop (timeout and re-issue): every
+    simulation, the per-tenant counts and re-issues, and two full logs."""
+    wl = W.make_workload(name, n_traces=nt, n_queries=nq)
+    sim = gpu(wl, record=[0, wl.n_sims - 1])
+    assert sim.info()["generic_kernel"] == 1
+    o, oe = oracle.run(wl, range(wl.n_sims), procs=NPROC, extra=True)
+    assert_same(sim.results(), o, name)
+    assert_extras(sim.extras(), oe, name)
+    if name == "faulty":
+        assert int(oe["reissued"].sum()) > 0
+    assert_logs(sim, wl, 0)
+    assert_logs(sim, wl, 1)
+    check_best(sim, wl, o)
+    sim.close()
+
+
+def test_single_shots_on_the_lean_kernel():
+    """Single-shot requests (k = 0) of one tenant run on the lean kernel."""
+    src = W.make_workload("competing-25", n_traces=2, n_queries=300)
+    traces = [W.Trace(*[getattr(t, f) for f in ("arrival_us", "k", "call_base", "prompt", "out", "out_est",
+                                                "stage", "cand", "retry")]) for t in src.traces]
+    c = src.cluster
+    cl = W.Cluster(c.prefill_tok_s, c.decode_us_tok, c.slots, c.inst_type, c.ref_type, c.slo_mult_fp, c.rmax,
+                   c.stage_ref_prompt, c.stage_ref_out)
+    wl = W.Workload("competing-25 one tenant", traces, cl, src.grid, src.objective)
+    assert (traces[0].k == 0).any()
+    sim = gpu(wl)
+    assert sim.info()["generic_kernel"] == 0
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(sim.results(), o, "lean single shots")
+    e = sim.extras()
+    assert (e["n_done"][:, 0] == o["n_done"]).all() and (e["n_done"][:, 1:] == 0).all()
+    sim.close()

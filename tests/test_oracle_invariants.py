@@ -21,6 +21,8 @@ def _release_times(tr, end):
     for i in range(tr.n_queries):
         b, e = int(tr.call_base[i]), int(tr.call_base[i + 1])
         rel[b] = tr.arrival_us[i]
+        if tr.k[i] == 0:
+            continue  # a single-shot request: one call, released on arrival
         last_of_chain = {}
         for j in range(b + 1, e - 1):
             c = int(tr.cand[j])
@@ -41,15 +43,37 @@ def _mix64(z):
     return z ^ (z >> 31)
 
 
-def check_schedule(tr, cl, res, log):
+def _slowdown(cl, inst, start):
+    """slow_fp of the first fault window covering each (instance, start), else 0."""
+    slow = np.zeros(inst.shape[0], np.int64)
+    hit = np.zeros(inst.shape[0], bool)
+    if cl.faults is not None:
+        for f in cl.faults:
+            sel = ~hit & (inst == f["inst"]) & (start >= f["t0_us"]) & (start < f["t1_us"])
+            slow[sel] = f["slow_fp"]
+            hit |= sel
+    return hit, slow
+
+
+def check_schedule(tr, cl, res, log, reissued=0):
+    """With re-issues the log keeps each call's last attempt only: the failed
+    attempts' slot time and digest terms are not in it, so work conservation
+    and the digest are checked only when nothing was re-issued."""
     p = oracle.prep(tr, cl)
     inst, enq, start, end = log["inst"], log["enq"], log["start"], log["end"]
     assert (inst >= 0).all() and (start >= 0).all()
     rel = _release_times(tr, end)
-    assert (enq == rel).all(), "dispatch must happen when the predecessors finish"
+    if reissued:
+        assert (enq >= rel).all()
+    else:
+        assert (enq == rel).all(), "dispatch must happen when the predecessors finish"
     assert (start >= enq).all()
     types = cl.inst_type[inst]
-    assert (end - start == p["svc"][np.arange(tr.n_calls), types]).all()
+    svc = p["svc"][np.arange(tr.n_calls), types]
+    hit, slow = _slowdown(cl, inst, start)
+    assert (slow[hit] > 0).all(), "no attempt that finished started on a stopped instance"
+    want = np.where(hit, -(-svc * slow // W.SCALE), svc)
+    assert (end - start == want).all()
     for m in range(cl.n_inst):
         slots = int(cl.slots[cl.inst_type[m]])
         on = np.nonzero(inst == m)[0]
@@ -59,6 +83,8 @@ def check_schedule(tr, cl, res, log):
         # running count after all events at time t
         running = np.array([np.sum((start[on] <= t) & (end[on] > t)) for t in times])
         assert running.max() <= slots
+        if reissued:
+            continue
         for c in on[start[on] > enq[on]]:
             sel = (times >= enq[c]) & (times < start[c])
             assert (running[sel] == slots).all(), "a call waited while a slot was free"
@@ -70,6 +96,8 @@ def check_schedule(tr, cl, res, log):
         assert int(res["p95_us"]) == int(np.sort(lat)[rank - 1])
         assert int(res["slo_met"]) == int(np.sum(lat <= p["t_slo"]))
         assert int(res["makespan_us"]) == int(end.max())
+    if reissued:
+        return
     gold, mixc, m64 = 0x9E3779B97F4A7C15, 0xBF58476D1CE4E5B9, (1 << 64) - 1
 
     def term(t, idtag):
@@ -161,3 +189,86 @@ def test_invariants_extra_recipes(name):
         res, log = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, p), check=True, log=True)
         assert res["status"] == 0
         check_schedule(tr, wl.cluster, res, log)
+
+
+@pytest.mark.parametrize("name", ["two-tenant", "competing-25", "competing-50"])
+def test_tenants_and_single_shots(name):
+    """Per-tenant SLO counts add up and match each tenant's own T_slo; the
+    single-shot requests (k = 0) run as one call released on arrival."""
+    wl = W.make_workload(name, n_traces=1, n_queries=150)
+    tr = wl.traces[0]
+    p = oracle.prep(tr, wl.cluster)
+    lat_ok = None
+    for pt_i in [0, wl.grid.n_points // 2, wl.grid.n_points - 1]:
+        res, log, ext = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, pt_i), check=True, log=True,
+                                        extra=True)
+        assert res["status"] == 0 and int(ext["reissued"]) == 0
+        check_schedule(tr, wl.cluster, res, log)
+        lat = log["end"][tr.call_base[1:] - 1] - tr.arrival_us
+        for t in range(4):
+            sel = tr.tenant == t
+            assert int(ext["n_done"][t]) == int(sel.sum())
+            assert int(ext["slo_met"][t]) == int(np.sum(lat[sel] <= p["t_slo"][sel]))
+        assert int(ext["slo_met"].sum()) == int(res["slo_met"])
+    if name.startswith("competing"):
+        single = tr.k == 0
+        frac = float(name.split("-")[1]) / 100
+        assert int(single.sum()) == int(np.floor(frac * (tr.n_calls - single.sum()) + 0.5))
+        assert (tr.stage[tr.call_base[:-1][single]] == W.STAGE_E).all()
+        assert (np.diff(tr.call_base)[single] == 1).all()
+        assert (tr.tenant[single] == 1).all() and (tr.tenant[~single] == 0).all()
+
+
+def test_equal_tenant_slos_change_nothing():
+    """Tenants whose SLO multipliers all equal the cluster's give the one-tenant result."""
+    wl = W.make_workload(1, n_traces=1, n_queries=200)
+    tr = wl.traces[0]
+    tr2 = W.Trace(*[getattr(tr, f) for f in ("arrival_us", "k", "call_base", "prompt", "out", "out_est",
+                                             "stage", "cand", "retry")],
+                  (np.arange(tr.n_queries) % 3).astype(np.uint8))
+    cl = wl.cluster
+    cl2 = W.Cluster(cl.prefill_tok_s, cl.decode_us_tok, cl.slots, cl.inst_type, cl.ref_type, cl.slo_mult_fp,
+                    cl.rmax, cl.stage_ref_prompt, cl.stage_ref_out, np.full(3, cl.slo_mult_fp, np.int64))
+    for p in [0, 30, 63]:
+        a = oracle.simulate(tr, cl, oracle.point_of(wl.grid, p))
+        b, ext = oracle.simulate(tr2, cl2, oracle.point_of(wl.grid, p), extra=True)
+        assert a.tolist() == b.tolist()
+        assert ext["n_done"].tolist()[:3] == [int(np.sum(tr2.tenant == t)) for t in range(3)]
+
+
+def _with_faults(cl, faults, timeout_fp):
+    f = np.zeros(len(faults), W.FAULT_DTYPE)
+    for j, x in enumerate(faults):
+        f[j] = (x[0], 0, x[1], x[2], x[3])
+    return W.Cluster(cl.prefill_tok_s, cl.decode_us_tok, cl.slots, cl.inst_type, cl.ref_type, cl.slo_mult_fp,
+                     cl.rmax, cl.stage_ref_prompt, cl.stage_ref_out, None, timeout_fp, f)
+
+
+def test_neutral_faults_change_nothing():
+    """An empty window, or a 1x slow-down without a timeout, is no fault."""
+    wl = W.make_workload(1, n_traces=1, n_queries=200)
+    tr, cl = wl.traces[0], wl.cluster
+    for faults, to in (([(0, 5_000_000, 5_000_000, 0)], 3 * W.SCALE), ([(1, 0, 10 ** 9, W.SCALE)], 0)):
+        cl2 = _with_faults(cl, faults, to)
+        for p in [0, 40, 63]:
+            a = oracle.simulate(tr, cl, oracle.point_of(wl.grid, p))
+            b, ext = oracle.simulate(tr, cl2, oracle.point_of(wl.grid, p), extra=True)
+            assert a.tolist() == b.tolist() and int(ext["reissued"]) == 0
+
+
+@pytest.mark.parametrize("dispatch", [W.DISPATCH_WB, W.DISPATCH_RR])
+def test_faulty_recipe_reissues(dispatch):
+    """Timeouts on slow or stopped instances re-issue requests elsewhere; every
+    call still completes once, and no finished attempt started on a stopped
+    instance inside its window."""
+    wl = W.make_workload("faulty", n_traces=1, n_queries=1400)
+    tr = wl.traces[0]
+    total = 0
+    for p in [0, 33, 63]:
+        pt = oracle.point_of(wl.grid, p)
+        pt["dispatch_policy"] = dispatch
+        res, log, ext = oracle.simulate(tr, wl.cluster, pt, check=True, log=True, extra=True)
+        assert res["status"] == 0
+        check_schedule(tr, wl.cluster, res, log, reissued=int(ext["reissued"]))
+        total += int(ext["reissued"])
+    assert total > 0

@@ -14,7 +14,7 @@ HAND = sorted(cases.load_golden("hand_cases.json")["cases"].keys())
 @pytest.mark.parametrize("name", HAND)
 def test_hand_case(name):
     tr, cl, exp = cases.hand_case(name)
-    res, log = oracle.simulate(tr, cl, exp["point"], check=True, log=True)
+    res, log, ext = oracle.simulate(tr, cl, exp["point"], check=True, log=True, extra=True)
     assert res["status"] == 0
     assert log["inst"].tolist() == exp["inst"]
     assert log["start"].tolist() == exp["start"]
@@ -27,6 +27,10 @@ def test_hand_case(name):
     assert int(res["makespan_us"]) == exp["makespan_us"]
     assert int(res["n_done"]) == tr.n_queries
     assert int(res["events"]) == tr.n_calls
+    if "tenant_slo_met" in exp:
+        assert ext["slo_met"].tolist() == exp["tenant_slo_met"]
+        assert ext["n_done"].tolist() == exp["tenant_done"]
+        assert int(ext["reissued"]) == exp["reissued"]
 
 
 def test_table2_pick():

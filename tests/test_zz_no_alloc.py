@@ -29,6 +29,20 @@ def test_static_matches_handle_path_twice():
             assert (gp, gs, gslo) == (wp, ws, wslo)
 
 
+@pytest.mark.gpu
+@pytest.mark.parametrize("name,nq", [("competing-25", 300), ("faulty", 1400)])
+def test_static_handles_tenants_single_shots_and_faults(name, nq):
+    B.build()
+    wl = W.make_workload(name, n_traces=1, n_queries=nq)
+    sim = H.Sim(wl.traces, wl.cluster, wl.grid)
+    sim.run()
+    want = sim.results()
+    sim.close()
+    got, _ = H.run_static(wl.traces[0], wl.cluster, wl.grid, W.OBJ_P95)
+    for f in FIELDS:
+        assert np.array_equal(got[f], want[f]), f
+
+
 def test_static_rejects_a_trace_that_does_not_fit():
     B.build()
     r = W.CONFIGS[4]
