@@ -791,13 +791,15 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             if (lane == 0) log_dispatch(a, recj, rid, m, now, budget);
           }
         }
-        if (rel_count == 1) {
-          // the event's only dispatch meets an empty queue and a free slot: it
-          // starts now, as the batch boundary below would start it
+        if (npend == 0) {
+          // nothing of this event waits yet, m's queue is empty and m has a
+          // free slot for this request and every one still to be dispatched in
+          // this event: the batch boundary below would start it now whatever
+          // the others do, so it starts at once
           uint64_t* const sl = W->slot + c.slot_base[m];
           __syncwarp();
           const int cn = W->cnt[m];
-          if (W->hsize[m] == 0 && cn < c.inst_slots[m]) {
+          if (W->hsize[m] == 0 && cn + (rel_count - jr) <= c.inst_slots[m]) {
             start_call(sl, m, cn, rid, svc_m);
             if (lane == 0) W->cnt[m] = cn + 1;
             set_key(m, sl[0]);
