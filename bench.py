@@ -197,8 +197,15 @@ def run_gpu(args):
     from paper_2505_05286_gb300 import build as B
     from paper_2505_05286_gb300 import hxsim as H
     B.build()
-    # weak scaling: every rank simulates its own 256 traces (trace seeds offset by rank)
-    wl = W.make_workload(CFG, first_trace=D.first_trace(rank, W.CONFIGS[CFG].n_traces))
+    # weak scaling: every rank simulates its own 256 traces (trace seeds offset by rank);
+    # --traces / --queries cut the workload down for profiling captures
+    nt = args.traces or W.CONFIGS[CFG].n_traces
+    wl = W.make_workload(CFG, n_traces=args.traces, n_queries=args.queries, first_trace=D.first_trace(rank, nt))
+    if args.alpha != "all":
+        # profiling: only the alpha = 1 points, or only the others
+        keep = (wl.grid.alpha_fp == W.SCALE) if args.alpha == "1" else (wl.grid.alpha_fp != W.SCALE)
+        wl = W.Workload(f"{wl.name}[alpha {args.alpha}]", wl.traces, wl.cluster,
+                        W.subset_grid(wl.grid, np.nonzero(keep)[0]), wl.objective)
     n_calls = wl.n_calls
     P = wl.grid.n_points
     sim = H.Sim(wl.traces, wl.cluster, wl.grid, timing=True)
@@ -276,7 +283,7 @@ def run_gpu(args):
             "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic",
             "stage_events_per_s": events_rate, "all_sims_ok": ok,
-            "config": {"workload": wl.name, "traces": len(wl.traces), "queries_per_trace": W.CONFIGS[CFG].n_queries,
+            "config": {"workload": wl.name, "traces": len(wl.traces), "queries_per_trace": wl.traces[0].n_queries,
                        "instances": n_inst, "points": P, "sims": wl.n_sims, "calls": n_calls,
                        "l2": f"inputs larger than L2 ({n_calls * 64 / 2**30:.2f} GiB of call records)",
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
@@ -303,6 +310,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--traces", type=int, default=None, help="cut the workload to this many traces (profiling)")
+    ap.add_argument("--queries", type=int, default=None, help="cut each trace to this many queries (profiling)")
+    ap.add_argument("--alpha", default="all", choices=["all", "1", "lt1"],
+                    help="profiling: keep only the alpha = 1 grid points, or only the others")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
