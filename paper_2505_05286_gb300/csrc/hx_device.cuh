@@ -162,7 +162,6 @@ struct WarpShared {
   int32_t n_done, slo_met, events, tk;
   int64_t tkmin;                // root of the full top-K heap (written alike by every lane)
   longlong2 dterm[16];          // digest terms waiting to be hashed: (time, id tag)
-  int32_t dn, pad1;             // terms waiting (written alike by every lane)
   int32_t tslo[HX_MAX_TENANTS], tdone[HX_MAX_TENANTS];  // per-tenant counts (generic kernel)
   int32_t reissued, excl;       // timed-out attempts; the instance a re-issue avoids (-1: none)
   uint64_t slot[1];             // [total_slots], then with faults one fail flag byte per slot

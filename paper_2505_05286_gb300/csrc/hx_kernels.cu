@@ -219,15 +219,15 @@ __device__ __noinline__ void digest_flush(WarpShared* W, int n, int lane) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) y += __shfl_xor_sync(kFull, y, o);
   if (lane == 0) W->digest += y;
-  W->dn = 0;
   __syncwarp();
 }
 
-__device__ __forceinline__ void digest_push(WarpShared* W, int64_t t, uint32_t tag, int lane) {
-  const int n = W->dn;
-  if (lane == 0) W->dterm[n] = make_longlong2(t, (long long)tag);
-  if (n == 15) digest_flush(W, 16, lane);
-  else W->dn = n + 1;
+__device__ __forceinline__ void digest_push(WarpShared* W, int& dn, int64_t t, uint32_t tag, int lane) {
+  if (lane == 0) W->dterm[dn] = make_longlong2(t, (long long)tag);
+  if (++dn == 16) {
+    digest_flush(W, 16, lane);
+    dn = 0;
+  }
 }
 
 __device__ __forceinline__ bool ent_better(long long ka, int ra, long long kb, int rb) {
@@ -436,14 +436,14 @@ __device__ __noinline__ int2 push_pop(WarpShared* W, const CallRec* rec, int64_t
 }
 
 // All lanes: a query's evaluation call finished at `now` (Sec. 4.3's metrics).
-__device__ __forceinline__ void finish_query(WarpShared* W, int32_t qid, int64_t now, int64_t arrival,
+__device__ __forceinline__ void finish_query(WarpShared* W, int& dn, int32_t qid, int64_t now, int64_t arrival,
                                             int64_t deadline, int lane) {
   if (lane == 0) {
     W->slo_met += now <= deadline ? 1 : 0;
     W->n_done++;
     W->makespan = now;
   }
-  digest_push(W, now, query_tag(qid), lane);
+  digest_push(W, dn, now, query_tag(qid), lane);
   // most latencies of a full heap fall below its root and change nothing
   const int64_t v = now - arrival;
   if (W->tk < W->kcap || v > W->tkmin) topk_insert_warp(W, v, lane);
@@ -552,7 +552,6 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       W->rr = 0;
       W->bump = 0;
       W->digest = 0;
-      W->dn = 0;
       W->makespan = 0;
       W->n_done = 0;
       W->slo_met = 0;
@@ -594,6 +593,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
 
     // Request rid starts on instance m now and runs until now + svc: its key
     // joins the cn sorted keys of m's running calls at sl.
+    int dn = 0;  // digest terms waiting in W->dterm
     auto start_call = [&](uint64_t* sl, int m, int cn, int rid, int svc) {
       int64_t run = svc;
       bool fail = false;
@@ -628,7 +628,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         if (lane >= pos && lane < cn) fl[lane + 1] = fcur;
         if (lane == pos) fl[pos] = fail ? 1 : 0;
       }
-      digest_push(W, now, call_tag(rid, m), lane);
+      digest_push(W, dn, now, call_tag(rid, m), lane);
       if (kGeneric && lane == 0) {
         const int recj = W->recj;
         if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
@@ -708,7 +708,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             W->tdone[ten]++;
             W->tslo[ten] += now <= dl ? 1 : 0;
           }
-          finish_query(W, qid, now, r->arrival, dl, lane);
+          finish_query(W, dn, qid, now, r->arrival, dl, lane);
         } else {
           const int32_t nx = tail.y;
           if (nx >= 0) {
@@ -872,7 +872,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       if (status != HX_OK) break;
     }
 
-    digest_flush(W, W->dn, lane);
+    digest_flush(W, dn, lane);
     if (lane == 0) {
       int st = status;
       const int32_t n_done = W->n_done;
