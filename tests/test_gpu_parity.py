@@ -375,3 +375,77 @@ def test_single_shots_on_the_lean_kernel():
     e = sim.extras()
     assert (e["n_done"][:, 0] == o["n_done"]).all() and (e["n_done"][:, 1:] == 0).all()
     sim.close()
+
+
+def _fault_cluster(c, faults, timeout_fp, tmult=None):
+    f = np.zeros(len(faults), W.FAULT_DTYPE)
+    for j, x in enumerate(faults):
+        f[j] = (x[0], 0, x[1], x[2], x[3])
+    return W.Cluster(c.prefill_tok_s, c.decode_us_tok, c.slots, c.inst_type, c.ref_type, c.slo_mult_fp, c.rmax,
+                     c.stage_ref_prompt, c.stage_ref_out, tmult, timeout_fp, f)
+
+
+def test_fault_edge_cases():
+    """Overlapping windows (the first listed applies), a window stopping two
+    instances at once, round robin stepping past the failed instance, and a
+    one-instance cluster where a re-issue returns to the same instance."""
+    src = W.make_workload(1, n_traces=1, n_queries=400)
+    tr, c, g = src.traces[0], src.cluster, src.grid
+    faults = [(0, 10_000_000, 40_000_000, 2 * W.SCALE), (0, 0, 60_000_000, 0), (1, 5_000_000, 70_000_000, 0),
+              (6, 20_000_000, 30_000_000, 0), (2, 0, 100_000_000, 3 * W.SCALE // 2)]
+    cl = _fault_cluster(c, faults, 2 * W.SCALE)
+    pts = [0, 9, 27, 63]
+    lp = np.zeros(len(pts), np.uint8)
+    dp = np.array([0, 1, 0, 1], np.uint8)
+    grid = W.Grid(g.alpha_fp[pts], g.gamma_fp[pts], g.rho[pts], g.beta_us2[pts], lp, dp)
+    wl = W.Workload("fault edges", [tr], cl, grid, W.OBJ_P95)
+    sim = gpu(wl, record=[1, 2])
+    o, oe = oracle.run(wl, range(wl.n_sims), procs=NPROC, extra=True)
+    assert_same(sim.results(), o, "fault edges")
+    assert_extras(sim.extras(), oe, "fault edges")
+    assert int(oe["reissued"].sum()) > 0
+    assert_logs(sim, wl, 0)
+    assert_logs(sim, wl, 1)
+    sim.close()
+    # one instance: a re-issue goes back to it
+    one = W.Cluster(c.prefill_tok_s[:1], c.decode_us_tok[:1], c.slots[:1], np.zeros(1, np.uint8), 0, c.slo_mult_fp,
+                    c.rmax, c.stage_ref_prompt, c.stage_ref_out, None, 3 * W.SCALE,
+                    np.array([(0, 0, 0, 2_000_000, 0)], W.FAULT_DTYPE))
+    tr1 = W.make_workload(0, n_queries=40).traces[0]
+    wl1 = W.Workload("one instance", [tr1], one, grid, W.OBJ_P95)
+    sim = gpu(wl1)
+    o, oe = oracle.run(wl1, range(wl1.n_sims), extra=True)
+    assert_same(sim.results(), o, "one instance")
+    assert_extras(sim.extras(), oe, "one instance")
+    sim.close()
+
+
+def test_four_tenants_and_only_single_shots():
+    """Four tenants with random assignment, and a trace made only of
+    single-shot requests."""
+    src = W.make_workload(1, n_traces=2, n_queries=300)
+    c = src.cluster
+    cl = W.Cluster(c.prefill_tok_s, c.decode_us_tok, c.slots, c.inst_type, c.ref_type, c.slo_mult_fp, c.rmax,
+                   c.stage_ref_prompt, c.stage_ref_out, np.array([W.SCALE, 2 * W.SCALE, 3 * W.SCALE, 16 * W.SCALE]))
+    rng = np.random.default_rng(5)
+    traces = []
+    for t in src.traces:
+        t2 = W.Trace(*[getattr(t, f) for f in ("arrival_us", "k", "call_base", "prompt", "out", "out_est", "stage",
+                                               "cand", "retry")], rng.integers(0, 4, t.n_queries).astype(np.uint8))
+        traces.append(t2)
+    # single shots only: one E call per query
+    n = 500
+    arr = np.cumsum(rng.integers(0, 400_000, n)).astype(np.int64)
+    singles = W.Trace(arr, np.zeros(n, np.uint8), np.arange(n + 1, dtype=np.int32),
+                      rng.integers(100, 5000, n).astype(np.int32), rng.integers(10, 400, n).astype(np.int32),
+                      np.full(n, 200, np.int32), np.full(n, W.STAGE_E, np.uint8), np.zeros(n, np.uint8),
+                      np.zeros(n, np.uint8), rng.integers(0, 4, n).astype(np.uint8))
+    traces.append(singles)
+    wl = W.Workload("tenants", traces, cl, W.subset_grid(src.grid, [0, 20, 45, 63]), W.OBJ_P95_SLO95)
+    sim = gpu(wl, record=[wl.n_sims - 1])
+    o, oe = oracle.run(wl, range(wl.n_sims), procs=NPROC, extra=True)
+    assert_same(sim.results(), o, "tenants")
+    assert_extras(sim.extras(), oe, "tenants")
+    assert_logs(sim, wl, 0)
+    check_best(sim, wl, o)
+    sim.close()
