@@ -145,6 +145,7 @@ struct WarpShared {
   int32_t A, one_minus_a;        // alpha and 1 - alpha, fixed point
   int32_t rewards, pad2;          // 1 when dispatch scores need the reward term
   int64_t G, beta;
+  float betaf, pad3;            // beta as a float (the reward quotient's numerator)
   int64_t frest[kFRows];        // rest-of-path cost of the budget denominator by fcode
   int32_t lpol, dpol, recj, kcap, rr, bump;
   // this warp's scratch slices and the current trace's offsets

@@ -63,11 +63,12 @@ __device__ __forceinline__ float s64_to_float(int64_t x) {
   return x < 0 ? -u64_to_float((uint64_t)(-x)) : u64_to_float((uint64_t)x);
 }
 
-__device__ __forceinline__ uint64_t udiv_trial(uint64_t n, uint64_t d) {
+// nf = u64_to_float(n), given by a caller that divides one n many times.
+__device__ __forceinline__ uint64_t udiv_trial_f(uint64_t n, float nf, uint64_t d) {
   if (d == 1) return n;
   float rd;
   asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(rd) : "f"(u64_to_float(d)));
-  const float qf = u64_to_float(n) * rd;
+  const float qf = nf * rd;
   if (qf >= 1073741824.0f) return n / d;
   uint64_t q = (uint32_t)qf;
   int64_t r = (int64_t)(n - q * d);
@@ -84,6 +85,8 @@ __device__ __forceinline__ uint64_t udiv_trial(uint64_t n, uint64_t d) {
   }
   return q;
 }
+
+__device__ __forceinline__ uint64_t udiv_trial(uint64_t n, uint64_t d) { return udiv_trial_f(n, u64_to_float(n), d); }
 
 // Workload-balanced reward term of Eq. (score): beta / max(t_queue, 1), capped.
 __device__ __forceinline__ int64_t reward_of(int64_t beta, int64_t q) {
@@ -545,6 +548,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       W->rewards = (A != kScale && !(kGeneric && a.dpol[p] == HX_DISPATCH_RR)) ? 1 : 0;
       W->G = a.gamma[p];
       W->beta = a.beta[p];
+      W->betaf = u64_to_float((uint64_t)a.beta[p]);
       W->lpol = a.lpol[p];
       W->dpol = a.dpol[p];
       W->recj = a.rec_map ? a.rec_map[sim] : -1;
@@ -748,7 +752,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         while (__any_sync(kFull, dirty0 || dirty1)) {
           const bool rj = dirty0 || dirty1;
           const int64_t q = W->q[dirty0 ? m0 : m1];
-          const uint64_t res = udiv_trial(rj ? beta : 0ull, (rj && q > 1) ? (uint64_t)q : 1ull);
+          const uint64_t res = udiv_trial_f(rj ? beta : 0ull, rj ? W->betaf : 0.0f, (rj && q > 1) ? (uint64_t)q : 1ull);
           const int64_t orew =
               (int64_t)W->one_minus_a * (res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap);
           if (dirty0) { orew0 = orew; dirty0 = false; }
