@@ -199,7 +199,7 @@ def run_gpu(args):
     B.build()
     # weak scaling: every rank simulates its own 256 traces (trace seeds offset by rank);
     # --traces / --queries cut the workload down for profiling captures
-    nt = args.traces or W.CONFIGS[CFG].n_traces
+    nt = args.traces or W.RECIPES[CFG].n_traces
     wl = W.make_workload(CFG, n_traces=args.traces, n_queries=args.queries, first_trace=D.first_trace(rank, nt))
     if args.alpha != "all":
         # profiling: only the alpha = 1 points, or only the others

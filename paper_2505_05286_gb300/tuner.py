@@ -159,7 +159,7 @@ class OnlineTuner:
 def shift_trace(rates_qps: Sequence[float], seconds: Sequence[float], recipe: int = 0, seed: int = 0) -> W.Trace:
     """A trace whose Poisson rate steps through `rates_qps`, each for the
     matching number of seconds (the 5 -> 20 -> 5 QPS shift of Sec. 5.1)."""
-    r = W.CONFIGS[recipe]
+    r = W.RECIPES[recipe]
     parts = []
     t_off = 0
     for j, (rate, sec) in enumerate(zip(rates_qps, seconds)):

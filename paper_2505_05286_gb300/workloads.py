@@ -15,7 +15,7 @@ Uniform doubles are (x >> 11) * 2^-53.  Every draw is addressed by
 (stream, index), so traces are reproducible independently of generation
 order.
 
-The five workload recipes (`CONFIGS`) stand in for the paper's BIRD / Spider
+The five workload recipes (`RECIPES`) stand in for the paper's BIRD / Spider
 derived traces (Sec. 5.1), which are not available: Poisson or two-state MMPP
 query arrivals, per-stage token-length distributions (uniform or clipped
 lognormal), candidate counts k, error probability p and retry limit R.  The
@@ -270,7 +270,7 @@ TYPES_4 = [(5000, 35, 4), (9000, 22, 8), (12000, 15, 8), (20000, 10, 16)]
 _GAMMA4 = [SCALE // 2, SCALE, 3 * SCALE // 2, 2 * SCALE]
 _GAMMA8 = [(i + 1) * SCALE // 4 for i in range(8)]
 
-CONFIGS: List[Recipe] = [
+RECIPES: List[Recipe] = [
     Recipe("tiny-1x200q-4inst-16pt", 1, 200, "poisson", [2.0], 0.0, [4, 4], 0.3, 2,
            _UNIF_PROMPT, _UNIF_OUT, _UNIF_OUT_EST, _UNIF_REF_PROMPT,
            [TYPE_A, TYPE_B], [2, 2], 0, 3 * SCALE,
@@ -554,9 +554,9 @@ def make_grid(recipe: Recipe, local_policy: int = POLICY_PQ, dispatch_policy: in
 
 def make_workload(cfg_id, n_traces: Optional[int] = None, n_queries: Optional[int] = None,
                   first_trace: int = 0) -> Workload:
-    """Workload of recipe `cfg_id` (an index of CONFIGS or a key of EXTRA),
+    """Workload of recipe `cfg_id` (an index of RECIPES or a key of EXTRA),
     optionally with fewer traces or queries."""
-    r = CONFIGS[cfg_id] if isinstance(cfg_id, int) else EXTRA[cfg_id]
+    r = RECIPES[cfg_id] if isinstance(cfg_id, int) else EXTRA[cfg_id]
     if not isinstance(cfg_id, int):
         cfg_id = EXTRA_ID[cfg_id]
     nt = r.n_traces if n_traces is None else int(n_traces)

@@ -174,7 +174,7 @@ def test_overload_long_queues():
 
 
 def test_ragged_traces_and_empty():
-    r = W.CONFIGS[2]
+    r = W.RECIPES[2]
     traces = [W.make_trace(r, 2, 0, n_queries=0), W.make_trace(r, 2, 1, n_queries=1),
               W.make_trace(r, 2, 2, n_queries=3), W.make_trace(r, 2, 3, n_queries=700),
               W.make_trace(r, 2, 4, n_queries=0), W.make_trace(r, 2, 5, n_queries=37)]
@@ -195,7 +195,7 @@ def test_ragged_traces_and_empty():
 def test_largest_shapes():
     """64 instances of 16 slots (1024 slots per simulation), k = 8 candidates,
     up to 15 corrections per chain."""
-    r = W.CONFIGS[2]
+    r = W.RECIPES[2]
     r2 = W.Recipe("maxshape", 2, 120, "poisson", [3.0], 0.0, [8, 8], 0.85, 15, r.prompt, r.out, r.out_est,
                   r.ref_prompt, [W.TYPE_C, W.TYPE_A], [64, 0], 1, 3 * W.SCALE, 4, [W.SCALE, 4 * W.SCALE], [0, 15],
                   [(1, 1)], 300_000, W.OBJ_P95)

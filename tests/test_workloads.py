@@ -20,7 +20,7 @@ def trace_digest(tr):
 
 @pytest.mark.parametrize("cfg", range(5))
 def test_structure(cfg):
-    r = W.CONFIGS[cfg]
+    r = W.RECIPES[cfg]
     tr = W.make_trace(r, cfg, 0, n_queries=min(r.n_queries, 3000))
     cb = tr.call_base
     assert cb[0] == 0 and cb[-1] == tr.n_calls and (np.diff(cb) >= 3).all()
@@ -41,7 +41,7 @@ def test_structure(cfg):
 @pytest.mark.parametrize("cfg", [0, 2, 3])
 def test_calls_per_query_mean(cfg):
     """E[calls/query] = 1 + E[k] (1 + sum_{r=1..R} p^r) + 1."""
-    r = W.CONFIGS[cfg]
+    r = W.RECIPES[cfg]
     tr = W.make_trace(r, cfg, 1, n_queries=20000)
     ek = (r.k_range[0] + r.k_range[1]) / 2
     expect = 2 + ek * (1 + sum(r.p_err ** j for j in range(1, r.rmax + 1)))
@@ -50,7 +50,7 @@ def test_calls_per_query_mean(cfg):
 
 
 def test_poisson_rate():
-    r = W.CONFIGS[3]
+    r = W.RECIPES[3]
     tr = W.make_trace(r, 3, 5, n_queries=20000)
     rate = tr.n_queries / (tr.arrival_us[-1] / 1e6)
     assert abs(rate - r.rate_qps[0]) < 0.03 * r.rate_qps[0]
@@ -58,7 +58,7 @@ def test_poisson_rate():
 
 def test_token_ranges():
     for cfg in (0, 3):
-        r = W.CONFIGS[cfg]
+        r = W.RECIPES[cfg]
         tr = W.make_trace(r, cfg, 0, n_queries=2000)
         for s in range(4):
             sel = tr.stage == s
@@ -68,7 +68,7 @@ def test_token_ranges():
 
 
 def test_deterministic_and_seeded():
-    r = W.CONFIGS[1]
+    r = W.RECIPES[1]
     a = W.make_trace(r, 1, 3, n_queries=500)
     b = W.make_trace(r, 1, 3, n_queries=500)
     c = W.make_trace(r, 1, 4, n_queries=500)
@@ -84,12 +84,12 @@ def test_golden_trace_digest():
 
 
 def test_grid_layout():
-    g = W.make_grid(W.CONFIGS[4])
+    g = W.make_grid(W.RECIPES[4])
     assert g.n_points == 1024
     # row-major with alpha outermost, beta multiplier innermost
     assert g.alpha_fp[0] == 0 and g.alpha_fp[-1] == W.SCALE and g.alpha_fp[128] == W.SCALE // 7
     assert g.rho[:16].tolist() == [0, 0, 0, 0, 1, 1, 1, 1, 2, 2, 2, 2, 3, 3, 3, 3]
     assert g.beta_us2[:4].tolist() == [500_000 ** 2 // 4, 500_000 ** 2 // 2, 500_000 ** 2, 2 * 500_000 ** 2]
-    g0 = W.make_grid(W.CONFIGS[0])
+    g0 = W.make_grid(W.RECIPES[0])
     assert g0.alpha_fp.tolist()[::4] == [0, 333333, 666666, 1000000]
     assert g0.gamma_fp.tolist()[:4] == [500000, 1000000, 1500000, 2000000]

@@ -45,7 +45,7 @@ def test_static_handles_tenants_single_shots_and_faults(name, nq):
 
 def test_static_rejects_a_trace_that_does_not_fit():
     B.build()
-    r = W.CONFIGS[4]
+    r = W.RECIPES[4]
     tr = W.make_trace(r, 4, 0, n_queries=30000)  # ~227k calls: > 64 MiB of intermediates
     with pytest.raises(H.HxError) as e:
         H.run_static(tr, W.make_cluster(r), W.subset_grid(W.make_grid(r), [0, 1]), stream=0)

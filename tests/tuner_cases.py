@@ -18,5 +18,5 @@ def shift_scenario():
     """5 -> 20 -> 5 queries/s on the recipe-0 cluster (about 10 q/s of capacity),
     20-second windows."""
     tr = T.shift_trace([5.0, 20.0, 5.0], [60.0, 40.0, 60.0], recipe=0, seed=1)
-    cl = W.make_cluster(W.CONFIGS[0])
+    cl = W.make_cluster(W.RECIPES[0])
     return tr, cl, dict(window_us=20_000_000, min_queries=5, beta_us2=400_000 ** 2)
