@@ -257,8 +257,13 @@ class Sim:
     def run(self, stream=None):
         _check(self.lib, self.lib.hx_sim_run(self.h, _stream_handle(stream)))
 
-    def results(self) -> np.ndarray:
-        out = np.zeros(self.n_sims, RESULT_DTYPE)
+    def results(self, out: Optional[np.ndarray] = None) -> np.ndarray:
+        """One RESULT_DTYPE row per simulation; `out` (e.g. pinned host memory)
+        receives them when given."""
+        if out is None:
+            out = np.zeros(self.n_sims, RESULT_DTYPE)
+        elif out.dtype != RESULT_DTYPE or out.shape[0] < self.n_sims or not out.flags["C_CONTIGUOUS"]:
+            raise ValueError("out must be a contiguous RESULT_DTYPE array with a row per simulation")
         _check(self.lib, self.lib.hx_sim_results(self.h, _p(out), self.n_sims))
         return out
 
