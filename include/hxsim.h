@@ -239,10 +239,11 @@ int hx_best_of_sums(const int64_t* sum_p95, const int64_t* sum_slo_met, const in
                     int64_t n_queries_total, int32_t objective, hx_best* out);
 
 /* Per-call log of recorded simulation `rec_index` (position in
- * opt.record_sims): instance, dispatch time, SLO budget and start time of
- * every call of its trace.  Arrays are [n_calls] of that trace. */
+ * opt.record_sims): instance, dispatch time, SLO budget, start and end time
+ * of every call of its trace (its last attempt when attempts were
+ * re-issued).  Arrays are [n_calls] of that trace; any may be NULL. */
 int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us,
-                   int64_t* budget_us, int64_t* start_us, size_t n_calls);
+                   int64_t* budget_us, int64_t* start_us, int64_t* end_us, size_t n_calls);
 
 /* Per-call preparation output of trace `trace_index` after a run: Eq. (comp)
  * per type (est with the believed output, svc with the true output),

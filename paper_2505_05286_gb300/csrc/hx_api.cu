@@ -87,6 +87,7 @@ struct hx_sim {
   int64_t* d_rec_enq = nullptr;
   int64_t* d_rec_budget = nullptr;
   int64_t* d_rec_start = nullptr;
+  int64_t* d_rec_end = nullptr;
   std::vector<int32_t> record_sims;
   // launch shape
   int blocks = 0, resident_warps = 0, smem_per_block = 0;
@@ -482,7 +483,8 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
     const int64_t n = (int64_t)h->n_record * h->rec_stride;
     if ((rc = h->alloc(&h->d_rec_map, h->n_sims)) || (rc = h->alloc(&h->d_rec_inst, n)) ||
         (rc = h->alloc(&h->d_rec_enq, n)) || (rc = h->alloc(&h->d_rec_budget, n)) ||
-        (rc = h->alloc(&h->d_rec_start, n)) || (rc = upload(h->d_rec_map, map.data(), h->n_sims, s0)))
+        (rc = h->alloc(&h->d_rec_start, n)) || (rc = h->alloc(&h->d_rec_end, n)) ||
+        (rc = upload(h->d_rec_map, map.data(), h->n_sims, s0)))
       return bail(rc);
     if (cudaStreamSynchronize(s0) != cudaSuccess) return bail(fail(HX_ERR_CUDA, "record map upload failed"));
   }
@@ -571,6 +573,7 @@ int hx_sim_run(hx_sim* h, void* stream) {
   sa.rec_enq = h->d_rec_enq;
   sa.rec_budget = h->d_rec_budget;
   sa.rec_start = h->d_rec_start;
+  sa.rec_end = h->d_rec_end;
   sa.rec_stride = h->rec_stride;
   sa.extras = h->d_extras;
 
@@ -722,7 +725,7 @@ int hx_best_of_sums(const int64_t* sum_p95, const int64_t* sum_slo_met, const in
 }
 
 int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us, int64_t* budget_us,
-                   int64_t* start_us, size_t n_calls) {
+                   int64_t* start_us, int64_t* end_us, size_t n_calls) {
   if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
   if (rec_index < 0 || rec_index >= h->n_record) return fail(HX_ERR_INVALID, "rec_index out of range");
@@ -735,6 +738,7 @@ int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us,
   if (enq_us) HX_CUDA(cudaMemcpy(enq_us, h->d_rec_enq + o, n_calls * sizeof(int64_t), cudaMemcpyDeviceToHost));
   if (budget_us) HX_CUDA(cudaMemcpy(budget_us, h->d_rec_budget + o, n_calls * sizeof(int64_t), cudaMemcpyDeviceToHost));
   if (start_us) HX_CUDA(cudaMemcpy(start_us, h->d_rec_start + o, n_calls * sizeof(int64_t), cudaMemcpyDeviceToHost));
+  if (end_us) HX_CUDA(cudaMemcpy(end_us, h->d_rec_end + o, n_calls * sizeof(int64_t), cudaMemcpyDeviceToHost));
   return HX_OK;
 }
 
@@ -1010,6 +1014,7 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   sa.rec_enq = nullptr;
   sa.rec_budget = nullptr;
   sa.rec_start = nullptr;
+  sa.rec_end = nullptr;
   sa.rec_stride = 0;
   sa.extras = nullptr;
 

@@ -123,6 +123,7 @@ struct SimArgs {
   int64_t* rec_enq;
   int64_t* rec_budget;
   int64_t* rec_start;
+  int64_t* rec_end;
   int64_t rec_stride;
   hx_extra* extras;         // [n_sims] per-tenant counts and re-issues (generic kernel), or NULL
 };

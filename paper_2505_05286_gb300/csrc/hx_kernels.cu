@@ -635,7 +635,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       digest_push(W, dn, now, call_tag(rid, m), lane);
       if (kGeneric && lane == 0) {
         const int recj = W->recj;
-        if (recj >= 0) a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
+        if (recj >= 0) {
+          a.rec_start[(int64_t)recj * a.rec_stride + rid] = now;
+          a.rec_end[(int64_t)recj * a.rec_stride + rid] = now + run;
+        }
       }
       __syncwarp();
     };

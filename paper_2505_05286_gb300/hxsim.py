@@ -110,7 +110,7 @@ def load(path: Optional[str] = None):
     lib.hx_last_error.argtypes = []
     for name, args in [("hx_sim_create", [vp, i32, vp, vp, vp, vp]), ("hx_sim_upload", [vp, vp, i32, vp]),
                        ("hx_sim_run", [vp, vp]), ("hx_sim_results", [vp, vp, sz]),
-                       ("hx_sim_best", [vp, i32, vp]), ("hx_sim_records", [vp, i32, vp, vp, vp, vp, sz]),
+                       ("hx_sim_best", [vp, i32, vp]), ("hx_sim_records", [vp, i32, vp, vp, vp, vp, vp, sz]),
                        ("hx_sim_prep", [vp, i32, vp, vp, vp, vp, sz]), ("hx_sim_timings", [vp, vp, vp, vp]),
                        ("hx_sim_info", [vp, vp]), ("hx_sim_destroy", [vp]),
                        ("hx_sim_run_static", [vp, vp, vp, i32, vp, vp, vp]),
@@ -291,9 +291,9 @@ class Sim:
         t = self.record_sims[rec_index] // self.n_points
         n = self.n_calls[t]
         out = dict(inst=np.zeros(n, np.int32), enq=np.zeros(n, np.int64), budget=np.zeros(n, np.int64),
-                   start=np.zeros(n, np.int64))
+                   start=np.zeros(n, np.int64), end=np.zeros(n, np.int64))
         _check(self.lib, self.lib.hx_sim_records(self.h, int(rec_index), _p(out["inst"]), _p(out["enq"]),
-                                                 _p(out["budget"]), _p(out["start"]), n))
+                                                 _p(out["budget"]), _p(out["start"]), _p(out["end"]), n))
         return out
 
     def prep(self, trace_index: int) -> dict:

@@ -31,6 +31,12 @@ def jain_index(rates: Sequence[float]) -> float:
     return 1.0 if s2 == 0.0 else float(np.sum(x) ** 2 / (x.size * s2))
 
 
+def query_latencies(trace, records) -> np.ndarray:
+    """Latency of every query of a recorded simulation (`Sim.records`): the
+    end of its last call (the evaluation stage) minus its arrival."""
+    return np.asarray(records["end"])[np.asarray(trace.call_base)[1:] - 1] - np.asarray(trace.arrival_us)
+
+
 def tenant_p95(latency_us: Sequence[int], tenant: Optional[Sequence[int]], n_tenants: int) -> List[Optional[int]]:
     """Nearest-rank P95 (sorted L[ceil(0.95 n) - 1]) of each tenant's query
     latencies; None for a tenant without queries."""

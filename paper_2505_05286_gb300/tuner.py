@@ -101,10 +101,8 @@ def gpu_backend(trace: W.Trace, cluster: W.Cluster, grid: W.Grid):
         sim.run()
         res = sim.results()
         rec = sim.records(0)
-        prep = sim.prep(0)
-        e = trace.call_base[1:] - 1
-        svc = prep["svc"][e, cluster.inst_type[rec["inst"][e]]]
-        lat = rec["start"][e] + svc - trace.arrival_us
+        # a query ends when its evaluation call (its last call) ends
+        lat = rec["end"][trace.call_base[1:] - 1] - trace.arrival_us
         return res, lat
     finally:
         sim.close()

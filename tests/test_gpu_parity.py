@@ -48,7 +48,7 @@ def assert_logs(sim, wl, j):
     tr = wl.traces[s // P]
     _, lo = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, s % P), log=True)
     lg = sim.records(j)
-    for f in ("inst", "enq", "budget", "start"):
+    for f in ("inst", "enq", "budget", "start", "end"):
         bad = np.nonzero(lg[f] != lo[f])[0]
         assert bad.size == 0, f"sim {s}: {f} differs first at call {bad[:5].tolist()}"
 
@@ -449,3 +449,21 @@ def test_four_tenants_and_only_single_shots():
     assert_logs(sim, wl, 0)
     check_best(sim, wl, o)
     sim.close()
+
+
+def test_per_tenant_p95_from_records():
+    """Per-tenant P95 from a recorded simulation's call end times equals the
+    oracle's, also when fault windows stretch services."""
+    from paper_2505_05286_gb300 import tenants as T
+    for name, nq in (("two-tenant", 400), ("faulty", 1400)):
+        wl = W.make_workload(name, n_traces=1, n_queries=nq)
+        tr = wl.traces[0]
+        sim = gpu(wl, record=[5, 40])
+        for j, s in enumerate([5, 40]):
+            _, lo = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, s), log=True)
+            lat_g = T.query_latencies(tr, sim.records(j))
+            lat_o = lo["end"][tr.call_base[1:] - 1] - tr.arrival_us
+            assert (lat_g == lat_o).all()
+            nt = wl.cluster.n_tenants
+            assert T.tenant_p95(lat_g, tr.tenant, nt) == T.tenant_p95(lat_o, tr.tenant, nt)
+        sim.close()
