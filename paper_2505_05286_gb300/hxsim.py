@@ -267,6 +267,14 @@ class Sim:
         _check(self.lib, self.lib.hx_sim_results(self.h, _p(out), self.n_sims))
         return out
 
+    def results_tensors(self) -> dict:
+        """The results as one torch tensor per field (int64 / int32 / the
+        digest's 64 bits as int64), indexed by simulation."""
+        import torch
+        r = self.results()
+        return {f: torch.from_numpy(np.ascontiguousarray(r[f]).view(np.int64) if f == "digest"
+                                    else np.ascontiguousarray(r[f])) for f in RESULT_DTYPE.names}
+
     def extras(self) -> np.ndarray:
         """Per-tenant SLO hits and completed queries, and re-issued attempts, one row per sim."""
         out = np.zeros(self.n_sims, EXTRA_DTYPE)

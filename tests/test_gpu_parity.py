@@ -467,3 +467,13 @@ def test_per_tenant_p95_from_records():
             nt = wl.cluster.n_tenants
             assert T.tenant_p95(lat_g, tr.tenant, nt) == T.tenant_p95(lat_o, tr.tenant, nt)
         sim.close()
+
+
+def test_results_as_tensors():
+    wl = W.make_workload(0)
+    sim = gpu(wl)
+    r = sim.results()
+    t = sim.results_tensors()
+    assert set(t) == set(H.RESULT_DTYPE.names)
+    assert (t["p95_us"].numpy() == r["p95_us"]).all() and (t["digest"].numpy().view(np.uint64) == r["digest"]).all()
+    sim.close()
