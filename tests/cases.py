@@ -76,3 +76,59 @@ def uniform_single_instance(n, arrivals, svc_us=1000, slots=1):
                    np.array([slots], np.int32), np.array([0], np.uint8), 0, 3 * W.SCALE, 0,
                    np.ones(4, np.int32), np.ones(4, np.int32))
     return tr, cl
+
+
+def random_workload(seed):
+    """A small random but valid workload: any cluster shape, k from 0 to 8,
+    retries up to R, tenants, fault windows, mixed policies."""
+    rng = np.random.default_rng(1000 + seed)
+    T = int(rng.integers(1, 5))
+    N = int(rng.integers(1, 65))
+    prefill = rng.integers(500, 30000, T).astype(np.int32)
+    decode = rng.integers(1, 60, T).astype(np.int32)
+    slots = rng.integers(1, 17, T).astype(np.int32)
+    inst_type = np.sort(rng.integers(0, T, N)).astype(np.uint8)
+    rmax = int(rng.integers(0, 5))
+    n_ten = int(rng.integers(1, 5))
+    tmult = rng.integers(W.SCALE, 6 * W.SCALE, n_ten).astype(np.int64) if n_ten > 1 else None
+    faults = None
+    timeout = 0
+    if rng.random() < 0.5:
+        timeout = int(rng.integers(W.SCALE, 4 * W.SCALE))
+        nf = int(rng.integers(1, 5))
+        faults = np.zeros(nf, W.FAULT_DTYPE)
+        for j in range(nf):
+            t0 = int(rng.integers(0, 60_000_000))
+            faults[j] = (int(rng.integers(0, N)), 0, t0, t0 + int(rng.integers(0, 30_000_000)),
+                         0 if rng.random() < 0.4 else int(rng.integers(W.SCALE // 2, 4 * W.SCALE)))
+    cl = W.Cluster(prefill, decode, slots, inst_type, int(rng.integers(0, T)), int(rng.integers(W.SCALE, 5 * W.SCALE)),
+                   rmax, rng.integers(100, 3000, 4).astype(np.int32), rng.integers(10, 300, 4).astype(np.int32),
+                   tmult, timeout, faults)
+    nq = int(rng.integers(1, 120))
+    arrival = np.sort(rng.integers(0, 80_000_000, nq)).astype(np.int64)
+    ks, base, stage, cand, retry = [], [0], [], [], []
+    for _ in range(nq):
+        k = int(rng.integers(0, 9))
+        ks.append(k)
+        if k == 0:
+            stage.append(W.STAGE_E); cand.append(0); retry.append(0)
+        else:
+            stage.append(W.STAGE_S); cand.append(0); retry.append(0)
+            for cidx in range(k):
+                stage.append(W.STAGE_G); cand.append(cidx); retry.append(0)
+            for cidx in range(k):
+                for r in range(1, int(rng.integers(0, rmax + 1)) + 1):
+                    stage.append(W.STAGE_C); cand.append(cidx); retry.append(r)
+            stage.append(W.STAGE_E); cand.append(0); retry.append(0)
+        base.append(len(stage))
+    nc = len(stage)
+    tr = W.Trace(arrival, np.array(ks, np.uint8), np.array(base, np.int32),
+                 rng.integers(1, 8000, nc).astype(np.int32), rng.integers(0, 600, nc).astype(np.int32),
+                 rng.integers(0, 600, nc).astype(np.int32), np.array(stage, np.uint8), np.array(cand, np.uint8),
+                 np.array(retry, np.uint8), rng.integers(0, n_ten, nq).astype(np.uint8) if n_ten > 1 else None)
+    P = 6
+    grid = W.Grid(rng.integers(0, W.SCALE + 1, P).astype(np.int64), rng.integers(0, 4 * W.SCALE + 1, P).astype(np.int64),
+                  rng.integers(0, 4, P).astype(np.int32), rng.integers(0, 10 ** 12, P).astype(np.int64),
+                  rng.integers(0, 3, P).astype(np.uint8), rng.integers(0, 2, P).astype(np.uint8))
+    grid.alpha_fp[0], grid.alpha_fp[1] = 0, W.SCALE
+    return W.Workload(f"random {seed}", [tr], cl, grid, int(rng.integers(0, 2)))

@@ -272,3 +272,24 @@ def test_faulty_recipe_reissues(dispatch):
         check_schedule(tr, wl.cluster, res, log, reissued=int(ext["reissued"]))
         total += int(ext["reissued"])
     assert total > 0
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_invariants_random_workloads(seed):
+    """Random clusters, traces (k from 0 to 8), tenants, fault windows and
+    mixed policies: the schedule invariants and the per-tenant counts hold."""
+    from tests import cases
+    wl = cases.random_workload(seed)
+    tr = wl.traces[0]
+    p = oracle.prep(tr, wl.cluster)
+    for pt_i in range(wl.grid.n_points):
+        res, log, ext = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, pt_i), check=True, log=True,
+                                        extra=True)
+        assert res["status"] == 0
+        check_schedule(tr, wl.cluster, res, log, reissued=int(ext["reissued"]))
+        lat = log["end"][tr.call_base[1:] - 1] - tr.arrival_us
+        ten = tr.tenant if tr.tenant is not None else np.zeros(tr.n_queries, np.uint8)
+        for t in range(4):
+            sel = ten == t
+            assert int(ext["n_done"][t]) == int(sel.sum())
+            assert int(ext["slo_met"][t]) == int(np.sum(lat[sel] <= p["t_slo"][sel]))
