@@ -492,3 +492,14 @@ def test_random_small_workloads(seed):
     assert_logs(sim, wl, 0)
     check_best(sim, wl, o)
     sim.close()
+
+
+def test_command_line(capsys):
+    import json
+    from paper_2505_05286_gb300 import __main__ as cli
+    assert cli.main(["--recipe", "0"]) == 0
+    out = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    wl = W.make_workload(0)
+    o = oracle_results(wl, range(wl.n_sims))
+    gp, gs, _ = oracle.best(o, 1, wl.grid.n_points, [wl.traces[0].n_queries], W.OBJ_P95)
+    assert out["best_point"] == gp and out["sum_p95_us"] == gs and out["failed"] == 0
