@@ -6,6 +6,9 @@ reduction, on the ceiling workload (256 traces x 20000 queries, 64
 instances of 4 types, 1024 hyper-parameter points = 262144 simulations).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+    python bench.py --recipe faulty --traces 256        # another recipe
+    python bench.py --traces 64 --policy rr-fcfs        # a policy variant
+
 
 Prints one JSON line.  `value` is simulations per second over the timed
 steps (inputs resident in HBM; they are larger than L2, so no flush is
@@ -45,10 +48,44 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2505_05286_gb300", "csrc", "hx_kernels.cu
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "hx_sim_kernel_traffic.txt")
 
 
+# grid-wide policy overrides (Sec. 5.1's ablations and baselines): local queue, dispatch
+POLICIES = {"wb-pq": (W.POLICY_PQ, W.DISPATCH_WB), "wb-fcfs": (W.POLICY_FCFS, W.DISPATCH_WB),
+            "rr-pq": (W.POLICY_PQ, W.DISPATCH_RR), "rr-fcfs": (W.POLICY_FCFS, W.DISPATCH_RR),
+            "wb-llf": (W.POLICY_LLF, W.DISPATCH_WB)}
+
+
+def _recipe(arg: str):
+    return int(arg) if arg.isdigit() else arg
+
+
+def _workload(args, first_trace: int = 0):
+    """The benchmarked workload: a recipe, optionally cut (--traces,
+    --queries, --alpha) and with one policy on every grid point (--policy)."""
+    wl = W.make_workload(_recipe(args.recipe), n_traces=args.traces, n_queries=args.queries,
+                         first_trace=first_trace)
+    if args.alpha != "all":
+        # profiling: only the alpha = 1 points, or only the others
+        keep = (wl.grid.alpha_fp == W.SCALE) if args.alpha == "1" else (wl.grid.alpha_fp != W.SCALE)
+        wl = W.Workload(f"{wl.name}[alpha {args.alpha}]", wl.traces, wl.cluster,
+                        W.subset_grid(wl.grid, np.nonzero(keep)[0]), wl.objective)
+    if args.policy != "grid":
+        lp, dp = POLICIES[args.policy]
+        g = wl.grid
+        g = W.Grid(g.alpha_fp, g.gamma_fp, g.rho, g.beta_us2, np.full(g.n_points, lp, np.uint8),
+                   np.full(g.n_points, dp, np.uint8))
+        wl = W.Workload(f"{wl.name}[{args.policy}]", wl.traces, wl.cluster, g, wl.objective)
+    return wl
+
+
+def _is_ceiling(args) -> bool:
+    return (_recipe(args.recipe) == CFG and args.traces is None and args.queries is None
+            and args.alpha == "all" and args.policy == "grid")
+
+
 def _traffic_per_launch(n_sims: int):
-    """DRAM bytes (read + write) of one simulation-kernel launch from the
-    committed ncu capture, scaled to this launch's simulations; None when the
-    kernel source changed since the capture."""
+    """DRAM bytes (read + write) of one simulation-kernel launch on the
+    ceiling workload from the committed ncu capture, scaled to this launch's
+    simulations; None when the kernel source changed since the capture."""
     import hashlib
     try:
         kv = dict(line.strip().split("=", 1) for line in open(TRAFFIC_FILE) if "=" in line)
@@ -160,7 +197,7 @@ def run_reference(args):
     world, rank, _ = D.env()
     if rank != 0:
         return
-    wl = W.make_workload(CFG)
+    wl = _workload(args)
     procs = os.cpu_count() or 1
     per_step = max(procs, 16)
     for w in range(args.warmup):
@@ -199,13 +236,9 @@ def run_gpu(args):
     B.build()
     # weak scaling: every rank simulates its own 256 traces (trace seeds offset by rank);
     # --traces / --queries cut the workload down for profiling captures
-    nt = args.traces or W.RECIPES[CFG].n_traces
-    wl = W.make_workload(CFG, n_traces=args.traces, n_queries=args.queries, first_trace=D.first_trace(rank, nt))
-    if args.alpha != "all":
-        # profiling: only the alpha = 1 points, or only the others
-        keep = (wl.grid.alpha_fp == W.SCALE) if args.alpha == "1" else (wl.grid.alpha_fp != W.SCALE)
-        wl = W.Workload(f"{wl.name}[alpha {args.alpha}]", wl.traces, wl.cluster,
-                        W.subset_grid(wl.grid, np.nonzero(keep)[0]), wl.objective)
+    r = _recipe(args.recipe)
+    nt = args.traces or (W.RECIPES[r] if isinstance(r, int) else W.EXTRA[r]).n_traces
+    wl = _workload(args, first_trace=D.first_trace(rank, nt))
     n_calls = wl.n_calls
     P = wl.grid.n_points
     sim = H.Sim(wl.traces, wl.cluster, wl.grid, timing=True)
@@ -243,12 +276,12 @@ def run_gpu(args):
 
     # end to end through the C ABI from pinned host buffers: upload, run, read back
     e2e_steps = 1
-    fields = ("arrival_us", "k", "call_base", "prompt", "out", "out_est", "stage", "cand", "retry")
-    pinned = [W.Trace(*[torch.from_numpy(np.ascontiguousarray(getattr(t, f))).pin_memory().numpy() for f in fields])
-              for t in wl.traces]
+    fields = ("arrival_us", "k", "call_base", "prompt", "out", "out_est", "stage", "cand", "retry", "tenant")
+    pin = lambda a: None if a is None else torch.from_numpy(np.ascontiguousarray(a)).pin_memory().numpy()
+    pinned = [W.Trace(*[pin(getattr(t, f)) for f in fields]) for t in wl.traces]
     res_host = torch.empty(wl.n_sims * H.RESULT_DTYPE.itemsize, dtype=torch.uint8).pin_memory().numpy()
     res_host = res_host.view(H.RESULT_DTYPE)
-    h2d = sum(getattr(t, f).nbytes for t in pinned for f in fields)
+    h2d = sum(getattr(t, f).nbytes for t in pinned for f in fields if getattr(t, f) is not None)
     d2h = wl.n_sims * H.RESULT_DTYPE.itemsize
     _barrier(world)
     torch.cuda.synchronize()
@@ -259,7 +292,7 @@ def run_gpu(args):
         res2 = sim.results(out=res_host)
     torch.cuda.synchronize()
     e2e_s = D.max_over_ranks(time.perf_counter() - t0)
-    ok = ok and bool((res2["digest"] == res["digest"]).all())
+    e2e_same = bool((res2["digest"] == res["digest"]).all())
     e2e_value = sims_total * e2e_steps / e2e_s
     # best point of the whole job: per-point sums over every rank's traces
     sp, ss, sf = sim.point_sums()
@@ -279,17 +312,19 @@ def run_gpu(args):
     n_inst = wl.cluster.n_inst
     achieved = WARP_INST_PER_EVENT * events_per_step / (kern_ms / 1000.0)
     roofline = {"bound": "alu", "achieved": achieved / 1e9, "peak": peak / 1e9, "unit": "Gwarp-inst/s",
-                "frac": achieved / peak, "traffic": _traffic_per_launch(wl.n_sims),
+                "frac": achieved / peak, "traffic": _traffic_per_launch(wl.n_sims) if _is_ceiling(args) else None,
                 "work_per_event": WARP_INST_PER_EVENT, "events_per_launch": events_per_step,
                 "kernel": "hx_sim_kernel" if info["generic_kernel"] else "hx_sim_kernel_lean", "kernel_ms": kern_ms,
                 "peak_source": f"{sm_count} SMs x 4 schedulers x {sm_mhz:.0f} MHz ({peak_kind} sm_max_mhz)"}
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-            "stage_events_per_s": events_rate, "all_sims_ok": ok,
+            "stage_events_per_s": events_rate, "all_sims_ok": ok, "e2e_same_results": e2e_same,
             "config": {"workload": wl.name, "traces": len(wl.traces), "queries_per_trace": wl.traces[0].n_queries,
                        "instances": n_inst, "points": P, "sims": wl.n_sims, "calls": n_calls,
-                       "l2": f"inputs larger than L2 ({n_calls * 64 / 2**30:.2f} GiB of call records)",
+                       "l2": (f"inputs larger than L2 ({n_calls * 64 / 2**30:.2f} GiB of call records)"
+                              if n_calls * 64 > L2_BYTES else
+                              f"inputs fit in L2 ({n_calls * 64 / 2**20:.1f} MiB of call records), not flushed"),
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "resident_warps": info["resident_warps"], "blocks": info["blocks"]},
             "kernels_ms": {"prep": prep_ms, "simulate": kern_ms, "best": best_ms},
@@ -318,6 +353,10 @@ def main():
     ap.add_argument("--queries", type=int, default=None, help="cut each trace to this many queries (profiling)")
     ap.add_argument("--alpha", default="all", choices=["all", "1", "lt1"],
                     help="profiling: keep only the alpha = 1 grid points, or only the others")
+    ap.add_argument("--recipe", default=str(CFG),
+                    help="index of workloads.RECIPES or a key of workloads.EXTRA (default: the ceiling workload)")
+    ap.add_argument("--policy", default="grid", choices=["grid"] + sorted(POLICIES),
+                    help="one local-queue / dispatch policy on every grid point (default: the recipe's own)")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

@@ -207,7 +207,8 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
 
 /* Replace the trace contents of an existing handle with traces of the same
  * shapes (n_queries and n_calls per trace), copying host -> device on
- * `stream`; no allocation. */
+ * `stream`; no allocation.  A trace whose tenant pointer is NULL puts every
+ * query in tenant 0, as at create. */
 int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream);
 
 /* Enqueue the whole path on `stream` (a cudaStream_t, NULL = legacy default):

@@ -237,6 +237,30 @@ def test_repeat_runs_and_upload():
     fresh.close()
 
 
+def test_upload_with_tenants():
+    # two-tenant traces: re-uploading them reproduces every result; uploading
+    # them without tenant arrays makes every query tenant 0
+    wl = W.make_workload("two-tenant", n_traces=2, n_queries=300)
+    sim = gpu(wl)
+    a, ea = sim.results(), sim.extras()
+    fields = ("arrival_us", "k", "call_base", "prompt", "out", "out_est", "stage", "cand", "retry", "tenant")
+    sim.upload([W.Trace(*[None if getattr(t, f) is None else getattr(t, f).copy() for f in fields])
+                for t in wl.traces])
+    sim.run()
+    assert_same(sim.results(), a, "upload with tenants")
+    assert np.array_equal(sim.extras(), ea)
+    plain = [W.Trace(*[getattr(t, f) for f in fields[:-1]]) for t in wl.traces]
+    sim.upload(plain)
+    sim.run()
+    b, eb = sim.results(), sim.extras()
+    o, oe = oracle.run(W.Workload("no tenants", plain, wl.cluster, wl.grid, wl.objective), range(wl.n_sims),
+                       procs=NPROC, extra=True)
+    assert_same(b, o, "upload without tenants")
+    assert_extras(eb, oe, "upload without tenants")
+    assert (eb["n_done"][:, 1] == 0).all()
+    sim.close()
+
+
 # ------------------------------------------------------------------ full size
 @pytest.mark.parametrize("cfg,n_sample", [(1, None), (2, 48), (3, 24)])
 def test_full_recipes_sampled(cfg, n_sample):

@@ -1,6 +1,7 @@
 """The online tuning loop of Sec. 4.3 (cold start, sliding windows, one-sided
 t-test, sweep over alpha) with the oracle as the simulation backend."""
 import numpy as np
+import pytest
 
 from paper_2505_05286_gb300 import tuner as T
 from paper_2505_05286_gb300 import workloads as W
@@ -51,3 +52,24 @@ def test_loop_cold_start_trigger_and_argmin():
             assert r.new_alpha_fp == int(np.argmin(p95)) * W.SCALE // 10
         else:
             assert r.new_alpha_fp == r.alpha_fp
+
+
+def test_command_line_tuning_host_logic(capsys, monkeypatch):
+    # the command line's tuning mode, with the oracle standing in for the
+    # CUDA backend: same windows and decisions as the loop driven directly
+    import json
+    from paper_2505_05286_gb300 import __main__ as cli
+    monkeypatch.setattr(T, "gpu_backend", C.oracle_backend)
+    assert cli.main(["--tune", "5,20,5", "--seconds", "60,40,60", "--window-s", "20", "--recipe", "0",
+                     "--seed", "1"]) == 0
+    lines = [json.loads(x) for x in capsys.readouterr().out.strip().splitlines()]
+    tr, cl, kw = C.shift_scenario()
+    ref = T.OnlineTuner(cl, backend=C.oracle_backend, **kw).run(tr)
+    assert len(lines) == len(ref) + 1
+    for w, r in zip(lines, ref):
+        assert (w["window"], w["queries"], w["p95_us"], w["triggered"], w["p_value"]) == \
+               (r.index, r.n_queries, r.p95_us, r.triggered, r.p_value)
+        assert round(w["alpha"] * W.SCALE) == r.alpha_fp and round(w["new_alpha"] * W.SCALE) == r.new_alpha_fp
+    assert lines[-1]["tunings"] == sum(r.triggered for r in ref)
+    with pytest.raises(SystemExit):
+        cli.main(["--tune", "5,20", "--seconds", "1,2,3"])
