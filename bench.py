@@ -82,19 +82,28 @@ def _is_ceiling(args) -> bool:
             and args.alpha == "all" and args.policy == "grid")
 
 
+def _ncu_figures():
+    """Figures of the committed ncu captures of the simulation kernel on the
+    ceiling workload; {} when the kernel source changed since the capture."""
+    import hashlib
+    try:
+        kv = dict(line.strip().split("=", 1) for line in open(TRAFFIC_FILE)
+                  if "=" in line and not line.startswith("#"))
+        with open(KERNEL_SRC, "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()
+        return kv if kv.get("kernel_sha256") == sha else {}
+    except OSError:
+        return {}
+
+
 def _traffic_per_launch(n_sims: int):
     """DRAM bytes (read + write) of one simulation-kernel launch on the
     ceiling workload from the committed ncu capture, scaled to this launch's
     simulations; None when the kernel source changed since the capture."""
-    import hashlib
+    kv = _ncu_figures()
     try:
-        kv = dict(line.strip().split("=", 1) for line in open(TRAFFIC_FILE) if "=" in line)
-        with open(KERNEL_SRC, "rb") as f:
-            sha = hashlib.sha256(f.read()).hexdigest()
-        if kv.get("kernel_sha256") != sha:
-            return None
         return float(kv["dram_bytes_per_launch"]) * n_sims / float(kv["sims_per_launch"])
-    except (OSError, KeyError, ValueError):
+    except (KeyError, ValueError):
         return None
 
 
@@ -316,6 +325,12 @@ def run_gpu(args):
                 "work_per_event": WARP_INST_PER_EVENT, "events_per_launch": events_per_step,
                 "kernel": "hx_sim_kernel" if info["generic_kernel"] else "hx_sim_kernel_lean", "kernel_ms": kern_ms,
                 "peak_source": f"{sm_count} SMs x 4 schedulers x {sm_mhz:.0f} MHz ({peak_kind} sm_max_mhz)"}
+    if _is_ceiling(args):
+        # issue-slot use and executed instructions per event from the committed ncu capture
+        kv = _ncu_figures()
+        for key in ("issue_active_frac", "warp_inst_per_event", "threads_per_inst"):
+            if key in kv:
+                roofline["ncu_" + key] = float(kv[key])
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic",
