@@ -74,7 +74,10 @@ enum {
   HX_ERR_OOM = 3,        /* device or host allocation failed */
   HX_ERR_CAPACITY = 4,   /* a simulation outgrew its scratch (per-sim status) */
   HX_ERR_STEP_LIMIT = 5, /* a simulation exceeded its event bound (per-sim status) */
-  HX_ERR_STATE = 6       /* call out of order (e.g. results before run) */
+  HX_ERR_STATE = 6,      /* call out of order (e.g. results before run) */
+  HX_ERR_INVARIANT = 7,  /* a simulation broke a scheduler invariant (per-sim status;
+                            a library bug, never expected) */
+  HX_SKIPPED = 8         /* not in the run's subset (per-sim status) */
 };
 
 enum { HX_STAGE_S = 0, HX_STAGE_G = 1, HX_STAGE_C = 2, HX_STAGE_E = 3 };
@@ -162,6 +165,12 @@ typedef struct hx_options {
   int32_t timing;                   /* 1 = time each kernel with CUDA events */
   int32_t force_generic;            /* 1 = always use the simulation kernel built for
                                        mixed policies and logging (testing) */
+  int32_t n_subset;                 /* 0 = run every simulation */
+  const int32_t* sim_subset;        /* [n_subset] distinct sim indices to run, any order; the
+                                       others report HX_SKIPPED, and the best-point
+                                       reduction counts them as failed */
+  int32_t checked;                  /* 1 = also check the scheduler's invariants after every
+                                       event (runs the generic kernel) */
 } hx_options;
 
 /* Per-simulation result, index sim = trace * n_points + point. */
@@ -173,7 +182,8 @@ typedef struct hx_result {
                            and every query's (id, end) */
   int32_t slo_met;      /* queries with latency <= T_slo */
   int32_t n_done;       /* completed queries */
-  int32_t status;       /* HX_OK or HX_ERR_CAPACITY / HX_ERR_STEP_LIMIT */
+  int32_t status;       /* HX_OK, HX_ERR_CAPACITY, HX_ERR_STEP_LIMIT, HX_ERR_INVARIANT
+                           or HX_SKIPPED */
   int32_t cycles_k;     /* diagnostic: SM clock cycles / 1024 the simulation took
                            (saturated; varies from run to run) */
 } hx_result;

@@ -83,6 +83,10 @@ struct hx_sim {
   int32_t n_record = 0;
   int64_t rec_stride = 0;
   int32_t* d_rec_map = nullptr;
+  // run only these simulations, in work order (NULL: all of them)
+  int64_t* d_subset = nullptr;
+  int64_t n_work = 0;
+  bool checked = false;
   int32_t* d_rec_inst = nullptr;
   int64_t* d_rec_enq = nullptr;
   int64_t* d_rec_budget = nullptr;
@@ -348,6 +352,33 @@ void fill_cluster(const hx_cluster* cluster, hx::ClusterK& ck) {
   ck.smem_per_warp = per_warp_smem(base, cluster->n_faults > 0);
 }
 
+// The simulations of opt->sim_subset, checked (in range, distinct) and sorted
+// into the kernel's work order: trace-major, highest point first.
+int order_subset(const hx_options* opt, int32_t n_traces, int32_t n_points, std::vector<int64_t>* out) {
+  out->clear();
+  if (!opt || opt->n_subset == 0) return HX_OK;
+  if (opt->n_subset < 0) return fail(HX_ERR_INVALID, "n_subset < 0");
+  if (!opt->sim_subset) return fail(HX_ERR_INVALID, "sim_subset is NULL");
+  const int64_t n_sims = (int64_t)n_traces * n_points;
+  std::vector<int64_t> w((size_t)opt->n_subset);
+  for (int32_t i = 0; i < opt->n_subset; ++i) {
+    const int64_t s = opt->sim_subset[i];
+    if (s < 0 || s >= n_sims)
+      return fail(HX_ERR_INVALID, "sim_subset[" + std::to_string(i) + "] = " + std::to_string(s) + " is out of range");
+    const int64_t t = s / n_points, p = s - t * n_points;
+    w[i] = t * n_points + (n_points - 1 - p);
+  }
+  std::sort(w.begin(), w.end());
+  for (size_t i = 1; i < w.size(); ++i)
+    if (w[i] == w[i - 1]) return fail(HX_ERR_INVALID, "sim_subset lists a simulation twice");
+  out->resize(w.size());
+  for (size_t i = 0; i < w.size(); ++i) {
+    const int64_t t = w[i] / n_points;
+    (*out)[i] = t * n_points + (n_points - 1 - (w[i] - t * n_points));
+  }
+  return HX_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -367,6 +398,9 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   for (int t = 0; t < n_traces; ++t)
     if ((rc = validate_trace(&traces[t], t, cluster, min_prefill, max_decode))) return rc;
   if (opt && opt->n_record > 0 && !opt->record_sims) return fail(HX_ERR_INVALID, "record_sims is NULL");
+  if (opt && opt->checked != 0 && opt->checked != 1) return fail(HX_ERR_INVALID, "checked must be 0 or 1");
+  std::vector<int64_t> subset;
+  if ((rc = order_subset(opt, n_traces, grid->n_points, &subset))) return rc;
 
   hx_sim* h = new (std::nothrow) hx_sim();
   if (!h) return fail(HX_ERR_OOM, "host allocation failed");
@@ -390,6 +424,8 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   }
   h->n_q = q_off[n_traces];
   h->n_c = c_off[n_traces];
+  h->n_work = subset.empty() ? h->n_sims : (int64_t)subset.size();
+  h->checked = opt && opt->checked == 1;
   if (h->n_c >= (int64_t(1) << 31)) return bail(fail(HX_ERR_INVALID, "more than 2^31 calls in total"));
 
   // cluster constants (kernel parameter)
@@ -428,11 +464,15 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
       (rc = upload(h->d_lp, grid->local_policy, h->n_points, s0)) ||
       (rc = upload(h->d_dp, grid->dispatch_policy, h->n_points, s0)))
     return bail(rc);
+  if (!subset.empty() && ((rc = h->alloc(&h->d_subset, (int64_t)subset.size())) ||
+                          (rc = upload(h->d_subset, subset.data(), (int64_t)subset.size(), s0))))
+    return bail(rc);
 
   // the lean instantiation serves grids that are all workload-balanced
   // dispatch with the urgency queue, log nothing, count one tenant and have
   // no fault windows
-  h->generic = (opt && (opt->n_record > 0 || opt->force_generic)) || ck.n_tenants > 1 || ck.n_faults > 0;
+  h->generic = (opt && (opt->n_record > 0 || opt->force_generic)) || h->checked || ck.n_tenants > 1 ||
+               ck.n_faults > 0;
   for (int p = 0; p < grid->n_points && !h->generic; ++p)
     if (grid->local_policy[p] != HX_LOCAL_PQ || grid->dispatch_policy[p] != HX_DISPATCH_WB) h->generic = true;
   const void* kfn = h->generic ? (const void*)hx::hx_sim_kernel : (const void*)hx::hx_sim_kernel_lean;
@@ -544,6 +584,9 @@ int hx_sim_run(hx_sim* h, void* stream) {
   pa.n_traces = h->n_traces;
   pa.rec = h->d_rec;
   pa.work_counter = h->d_counter;
+  pa.skip_results = h->d_results;
+  pa.skip_extras = h->d_extras;
+  pa.n_skip = h->d_subset ? h->n_sims : 0;
 
   hx::SimArgs sa;
   sa.rec = h->d_rec;
@@ -576,6 +619,9 @@ int hx_sim_run(hx_sim* h, void* stream) {
   sa.rec_end = h->d_rec_end;
   sa.rec_stride = h->rec_stride;
   sa.extras = h->d_extras;
+  sa.subset = h->d_subset;
+  sa.n_work = h->n_work;
+  sa.checked = h->checked ? 1 : 0;
 
   hx::BestArgs ba;
   ba.results = h->d_results;
@@ -985,6 +1031,9 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   pa.n_traces = 1;
   pa.rec = static_cast<hx::CallRec*>(at(o_rec));
   pa.work_counter = static_cast<unsigned long long*>(at(o_ctr));  // zeroed by the prep kernel
+  pa.skip_results = nullptr;
+  pa.skip_extras = nullptr;
+  pa.n_skip = 0;
 
   hx::SimArgs sa;
   sa.rec = pa.rec;
@@ -1017,6 +1066,9 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   sa.rec_end = nullptr;
   sa.rec_stride = 0;
   sa.extras = nullptr;
+  sa.subset = nullptr;
+  sa.n_work = P;
+  sa.checked = 0;
 
   hx::BestArgs ba;
   ba.results = sa.results;

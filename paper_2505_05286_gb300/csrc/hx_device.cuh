@@ -93,6 +93,9 @@ struct PrepArgs {
   int32_t n_traces;
   CallRec* rec;             // [C]
   unsigned long long* work_counter;
+  hx_result* skip_results;  // with a subset: every result starts as HX_SKIPPED
+  hx_extra* skip_extras;    // and its per-tenant counts at zero (NULL: none kept)
+  int64_t n_skip;           // n_sims with a subset, else 0
 };
 
 struct SimArgs {
@@ -126,6 +129,9 @@ struct SimArgs {
   int64_t* rec_end;
   int64_t rec_stride;
   hx_extra* extras;         // [n_sims] per-tenant counts and re-issues (generic kernel), or NULL
+  const int64_t* subset;    // [n_work] sims to run in work order, or NULL: all n_sims
+  int64_t n_work;
+  int32_t checked;          // check the scheduler's invariants after every event (generic kernel)
 };
 
 // Per-warp shared memory of one simulation: per-instance local-queue and

@@ -113,6 +113,29 @@ __device__ __forceinline__ int64_t cost_on_type(const ClusterK& c, int t, int64_
 __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
   int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (g == 0) *a.work_counter = 0ull;
+  // a run over a subset: the simulations outside it report HX_SKIPPED
+  for (int64_t i = g; i < a.n_skip; i += (int64_t)gridDim.x * blockDim.x) {
+    hx_result r;
+    r.p95_us = -1;
+    r.makespan_us = 0;
+    r.events = 0;
+    r.digest = 0;
+    r.slo_met = 0;
+    r.n_done = 0;
+    r.status = HX_SKIPPED;
+    r.cycles_k = 0;
+    a.skip_results[i] = r;
+    if (a.skip_extras) {
+      hx_extra x;
+      for (int t = 0; t < HX_MAX_TENANTS; ++t) {
+        x.slo_met[t] = 0;
+        x.n_done[t] = 0;
+      }
+      x.reissued = 0;
+      x.pad = 0;
+      a.skip_extras[i] = x;
+    }
+  }
   if (g >= a.n_queries) return;
   int lo = 0, hi = a.n_traces;  // trace of query g: q_off[t] <= g < q_off[t+1]
   while (hi - lo > 1) {
@@ -489,11 +512,19 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     unsigned long long work = 0;
     if (lane == 0) work = atomicAdd(a.work_counter, 1ull);
     const int64_t w = (int64_t)__shfl_sync(kFull, work, 0);
-    if (w >= a.n_sims) break;
+    if (w >= a.n_work) break;
     // trace-major, so that concurrent simulations share a trace in L2; within a
     // trace the highest point index (highest alpha, the longest queues) first
-    const int t = (int)(w / a.n_points);
-    const int p = a.n_points - 1 - (int)(w - (int64_t)t * a.n_points);
+    // (a subset comes sorted in the same order)
+    int t, p;
+    if (a.subset) {
+      const int64_t s = a.subset[w];
+      t = (int)(s / a.n_points);
+      p = (int)(s - (int64_t)t * a.n_points);
+    } else {
+      t = (int)(w / a.n_points);
+      p = a.n_points - 1 - (int)(w - (int64_t)t * a.n_points);
+    }
     const int64_t sim = (int64_t)t * a.n_points + p;
     const long long clk0 = clock64();
     const int64_t qb = a.q_off[t];
@@ -876,19 +907,39 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         if (lane == 0) W->cnt[m] = cn;
         set_key(m, cn ? sl[0] : kKeyInf);
       }
+      if (kGeneric && a.checked && status == HX_OK) {
+        // after every event: no instance runs more calls than it has slots or
+        // keeps a slot free while requests wait in its queue (Sec. 4.2: free
+        // slots take waiting requests at every batch boundary), and t_queue
+        // stays non-negative
+        __syncwarp();
+        bool bad = false;
+        for (int m = lane; m < N; m += 32) {
+          const int cn = W->cnt[m], ns = c.inst_slots[m];
+          bad |= cn > ns || (cn < ns && W->hsize[m] > 0) || W->q[m] < 0;
+        }
+        if (__any_sync(kFull, bad)) status = HX_ERR_INVARIANT;
+      }
       if (status != HX_OK) break;
     }
 
     digest_flush(W, dn, lane);
+    // conservation at the end: every dispatched request finished (t_queue back
+    // to zero, no running call, no waiting request)
+    bool left = false;
+    for (int m = lane; m < N; m += 32) left |= W->q[m] != 0 || W->cnt[m] != 0 || W->hsize[m] != 0;
+    const bool leftover = __any_sync(kFull, left);
     if (lane == 0) {
       int st = status;
       const int32_t n_done = W->n_done;
-      if (st == HX_OK && n_done != nq) st = HX_ERR_STEP_LIMIT;
+      const int32_t steps0 = W->nc + nq + 8 + (kGeneric && c.n_faults > 0 ? 16 * W->nc + 4096 : 0);
+      const int64_t events = (steps0 - steps_left) - W->qa - (kGeneric ? W->reissued : 0);
+      // every query and every call completed exactly once
+      if (st == HX_OK && (leftover || n_done != nq || events != W->nc)) st = HX_ERR_INVARIANT;
       hx_result res;
       res.p95_us = st == HX_OK ? (nq > 0 ? W->topk[0] : 0) : -1;
       res.makespan_us = W->makespan;
-      const int32_t steps0 = W->nc + nq + 8 + (kGeneric && c.n_faults > 0 ? 16 * W->nc + 4096 : 0);
-      res.events = (steps0 - steps_left) - W->qa - (kGeneric ? W->reissued : 0);
+      res.events = events;
       res.digest = W->digest;
       res.slo_met = W->slo_met;
       res.n_done = n_done;

@@ -22,7 +22,8 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libhxsim.so")
 HEADER = os.path.join(os.path.dirname(_PKG), "include", "hxsim.h")
 
-HX_OK, HX_ERR_INVALID, HX_ERR_CUDA, HX_ERR_OOM, HX_ERR_CAPACITY, HX_ERR_STEP_LIMIT, HX_ERR_STATE = range(7)
+(HX_OK, HX_ERR_INVALID, HX_ERR_CUDA, HX_ERR_OOM, HX_ERR_CAPACITY, HX_ERR_STEP_LIMIT, HX_ERR_STATE,
+ HX_ERR_INVARIANT, HX_SKIPPED) = range(9)
 OBJ_P95, OBJ_P95_SLO95 = 0, 1
 
 RESULT_DTYPE = np.dtype([("p95_us", "<i8"), ("makespan_us", "<i8"), ("events", "<i8"),
@@ -69,7 +70,8 @@ class hx_grid(ctypes.Structure):
 class hx_options(ctypes.Structure):
     _fields_ = [("n_record", ctypes.c_int32), ("record_sims", ctypes.c_void_p),
                 ("max_resident_warps", ctypes.c_int32), ("timing", ctypes.c_int32),
-                ("force_generic", ctypes.c_int32)]
+                ("force_generic", ctypes.c_int32), ("n_subset", ctypes.c_int32), ("sim_subset", ctypes.c_void_p),
+                ("checked", ctypes.c_int32)]
 
 
 class hx_best(ctypes.Structure):
@@ -228,7 +230,11 @@ class Sim:
     """A set of (trace x point) simulations resident on the current CUDA device."""
 
     def __init__(self, traces, cluster, grid, record_sims: Sequence[int] = (), timing: bool = False,
-                 max_resident_warps: int = 0, force_generic: bool = False):
+                 max_resident_warps: int = 0, force_generic: bool = False, subset: Optional[Sequence[int]] = None,
+                 checked: bool = False):
+        """`subset`: run only these simulations (index trace * P + point); the
+        others report HX_SKIPPED.  `checked`: also check the scheduler's
+        invariants after every event (per-sim status HX_ERR_INVARIANT)."""
         self.lib = load()
         self.n_traces = len(traces)
         self.n_points = int(grid.alpha_fp.shape[0])
@@ -239,8 +245,10 @@ class Sim:
         hg, keep_g = _grid_struct(grid)
         self.record_sims = [int(s) for s in record_sims]
         rs = _c(self.record_sims if self.record_sims else [0], np.int32)
+        self.subset = None if subset is None else [int(s) for s in subset]
+        ss = _c(self.subset if self.subset else [0], np.int32)
         opt = hx_options(len(self.record_sims), _p(rs), int(max_resident_warps), int(bool(timing)),
-                         int(bool(force_generic)))
+                         int(bool(force_generic)), len(self.subset or []), _p(ss), int(bool(checked)))
         h = ctypes.c_void_p()
         _check(self.lib, self.lib.hx_sim_create(tr.arr, self.n_traces, ctypes.byref(hc), ctypes.byref(hg),
                                                 ctypes.byref(opt), ctypes.byref(h)))

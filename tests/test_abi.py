@@ -43,6 +43,7 @@ int main(void) {
   S(hx_extra) F(hx_extra, n_done) F(hx_extra, reissued)
   S(hx_grid) F(hx_grid, alpha_fp) F(hx_grid, dispatch_policy)
   S(hx_options) F(hx_options, record_sims) F(hx_options, timing) F(hx_options, force_generic)
+  F(hx_options, n_subset) F(hx_options, sim_subset) F(hx_options, checked)
   S(hx_result) F(hx_result, digest) F(hx_result, status) F(hx_result, cycles_k)
   S(hx_best) F(hx_best, global_sum_p95) F(hx_best, per_trace_point)
   S(hx_info) F(hx_info, resident_warps) F(hx_info, smem_per_block) F(hx_info, generic_kernel)
@@ -82,7 +83,7 @@ def test_struct_layout_matches_binding(tmp_path):
             assert ctypes.sizeof(structs[key]) == val[0], key
 
 
-def _create(lib, traces, cluster, grid):
+def _create(lib, traces, cluster, grid, opt=None):
     t = H._Traces(traces)
     hc, keep = H._cluster_struct(cluster)
     g = grid
@@ -91,7 +92,8 @@ def _create(lib, traces, cluster, grid):
           np.ascontiguousarray(g.local_policy, np.uint8), np.ascontiguousarray(g.dispatch_policy, np.uint8)]
     hg = H.hx_grid(len(gc[0]), *[H._p(x) for x in gc])
     h = ctypes.c_void_p()
-    rc = lib.hx_sim_create(t.arr, len(traces), ctypes.byref(hc), ctypes.byref(hg), None, ctypes.byref(h))
+    rc = lib.hx_sim_create(t.arr, len(traces), ctypes.byref(hc), ctypes.byref(hg),
+                           None if opt is None else ctypes.byref(opt), ctypes.byref(h))
     return rc, lib.hx_last_error().decode(), h
 
 
@@ -151,6 +153,26 @@ def test_rejects_malformed_inputs_without_device_work(lib):
     cases.append(("timeout < 1", [tr], faulty([(0, 0, 100, 0)], W.SCALE // 2), wl.grid, "timeout_mult_fp"))
     for name, trs, cl, gr, msg in cases:
         rc, err, h = _create(lib, trs, cl, gr)
+        assert rc == H.HX_ERR_INVALID, name
+        assert msg in err, (name, err)
+        assert not h.value
+
+
+def test_rejects_bad_subset_and_checked_flag(lib):
+    wl = W.make_workload(0, n_queries=20)  # 1 trace x 16 points
+
+    def opt(subset=None, n=None, checked=0):
+        arr = np.asarray(subset if subset else [0], np.int32)
+        o = H.hx_options(0, None, 0, 0, 0, len(subset or []) if n is None else n,
+                         None if subset is None else H._p(arr), checked)
+        return o, arr
+    for name, (o, keep), msg in [("out of range", opt([3, 16]), "out of range"),
+                                 ("negative index", opt([-1]), "out of range"),
+                                 ("twice", opt([5, 2, 5]), "twice"),
+                                 ("negative count", opt([1], n=-1), "n_subset"),
+                                 ("NULL subset", opt(None, n=2), "NULL"),
+                                 ("checked = 2", opt(None, n=0, checked=2), "checked")]:
+        rc, err, h = _create(lib, wl.traces, wl.cluster, wl.grid, o)
         assert rc == H.HX_ERR_INVALID, name
         assert msg in err, (name, err)
         assert not h.value

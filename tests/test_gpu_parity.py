@@ -527,3 +527,45 @@ def test_command_line(capsys):
     o = oracle_results(wl, range(wl.n_sims))
     gp, gs, _ = oracle.best(o, 1, wl.grid.n_points, [wl.traces[0].n_queries], W.OBJ_P95)
     assert out["best_point"] == gp and out["sum_p95_us"] == gs and out["failed"] == 0
+
+
+# ------------------------------------------------------------ subset, checked
+@pytest.mark.parametrize("generic", [False, True])
+def test_subset_runs_only_the_listed_simulations(generic):
+    wl = W.make_workload(1, n_traces=2, n_queries=300)  # 2 traces x 64 points
+    sub = [5, 64 + 63, 0, 64 + 7, 40, 63]
+    sim = gpu(wl, subset=sub, force_generic=generic)
+    r = sim.results()
+    inside = np.zeros(wl.n_sims, bool)
+    inside[sub] = True
+    o = oracle_results(wl, sub)
+    assert_same(r[np.sort(sub)], o[np.argsort(sub)], "subset")
+    assert (r["status"][~inside] == H.HX_SKIPPED).all() and (r["p95_us"][~inside] == -1).all()
+    assert (r["events"][~inside] == 0).all() and (r["n_done"][~inside] == 0).all()
+    if generic:
+        e = sim.extras()
+        assert (e["n_done"][~inside] == 0).all() and (e["n_done"][inside].sum(axis=1) == 300).all()
+    # the best-point reduction counts the skipped simulations as failed
+    check_best(sim, wl, r)
+    sim.run()
+    assert_same(sim.results(), r, "subset re-run")
+    sim.close()
+
+
+@pytest.mark.parametrize("name,nt,nq", [(1, 2, 300), ("faulty", 1, 1400), ("competing-50", 1, 300)])
+def test_checked_mode_changes_nothing(name, nt, nq):
+    """With the per-event invariant checks on (generic kernel), every
+    simulation still matches the oracle, status included."""
+    wl = W.make_workload(name, n_traces=nt, n_queries=nq)
+    if name == 1:
+        # mixed policies over the points
+        g = wl.grid
+        lp = np.array([W.POLICY_PQ, W.POLICY_FCFS, W.POLICY_LLF, W.POLICY_PQ], np.uint8)[np.arange(g.n_points) % 4]
+        dp = np.array([W.DISPATCH_WB, W.DISPATCH_WB, W.DISPATCH_WB, W.DISPATCH_RR], np.uint8)[np.arange(g.n_points) % 4]
+        wl = W.Workload(wl.name, wl.traces, wl.cluster, W.Grid(g.alpha_fp, g.gamma_fp, g.rho, g.beta_us2, lp, dp),
+                        wl.objective)
+    sim = gpu(wl, checked=True)
+    assert sim.info()["generic_kernel"] == 1
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(sim.results(), o, f"checked {name}")
+    sim.close()
