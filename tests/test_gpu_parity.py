@@ -506,9 +506,10 @@ def test_results_as_tensors():
 @pytest.mark.parametrize("seed", range(24))
 def test_random_small_workloads(seed):
     """Random clusters, traces and grids: every simulation, the per-tenant
-    counts and a full log equal the oracle's."""
+    counts and a full log equal the oracle's (odd seeds with the per-event
+    invariant checks on)."""
     wl = cases.random_workload(seed)
-    sim = gpu(wl, record=[wl.n_sims - 1])
+    sim = gpu(wl, record=[wl.n_sims - 1], checked=bool(seed % 2))
     o, oe = oracle.run(wl, range(wl.n_sims), extra=True)
     assert (o["status"] == 0).all()
     assert_same(sim.results(), o, wl.name)
