@@ -208,3 +208,26 @@ def test_best_point_rules():
     res["status"][1] = 2  # a failed simulation never wins
     gp, gs, per = oracle.best(res, 2, 3, [100, 100], W.OBJ_P95)
     assert per.tolist() == [2, 0] and gp == 0
+
+
+@pytest.mark.parametrize("alpha_index", [1, 3, 5])
+def test_wb_moves_work_to_fast_instances(alpha_index):
+    """Table 1 / Sec. 5.3, qualitatively: round robin spreads every stage over
+    the instances evenly, while workload-balanced dispatch sends a larger share
+    of each stage to the fastest instance type and a smaller one to the
+    slowest (recipe 1: 4 A, 2 B = slowest, 2 C = fastest)."""
+    wl = W.make_workload(1, n_traces=1, n_queries=500)
+    tr, cl = wl.traces[0], wl.cluster
+    pt = oracle.point_of(wl.grid, alpha_index * 8 + 3)
+    assert 0 < pt["alpha_fp"] < W.SCALE
+    rr = dict(pt, dispatch_policy=W.DISPATCH_RR)
+    _, wb_log = oracle.simulate(tr, cl, pt, log=True)
+    _, rr_log = oracle.simulate(tr, cl, rr, log=True)
+    inst_share = np.bincount(cl.inst_type, minlength=3) / cl.n_inst
+    fast, slow = 2, 1
+    for st in range(4):
+        sel = tr.stage == st
+        wb = np.bincount(cl.inst_type[wb_log["inst"][sel]], minlength=3) / sel.sum()
+        rrs = np.bincount(cl.inst_type[rr_log["inst"][sel]], minlength=3) / sel.sum()
+        assert np.abs(rrs - inst_share).max() < 0.05, (st, rrs)
+        assert wb[fast] > rrs[fast] + 0.1 and wb[slow] < rrs[slow] - 0.1, (st, wb, rrs)
