@@ -171,6 +171,9 @@ typedef struct hx_options {
                                        reduction counts them as failed */
   int32_t checked;                  /* 1 = also check the scheduler's invariants after every
                                        event (runs the generic kernel) */
+  int32_t arena_entries;            /* testing: local-queue entries per resident warp
+                                       (0 = enough for any run); a simulation whose
+                                       queues outgrow it reports HX_ERR_CAPACITY */
 } hx_options;
 
 /* Per-simulation result, index sim = trace * n_points + point. */

@@ -399,6 +399,7 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
     if ((rc = validate_trace(&traces[t], t, cluster, min_prefill, max_decode))) return rc;
   if (opt && opt->n_record > 0 && !opt->record_sims) return fail(HX_ERR_INVALID, "record_sims is NULL");
   if (opt && opt->checked != 0 && opt->checked != 1) return fail(HX_ERR_INVALID, "checked must be 0 or 1");
+  if (opt && opt->arena_entries < 0) return fail(HX_ERR_INVALID, "arena_entries < 0");
   std::vector<int64_t> subset;
   if ((rc = order_subset(opt, n_traces, grid->n_points, &subset))) return rc;
 
@@ -498,6 +499,7 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   // heap arena: doubling regions of 16, 32, ... entries per instance total at
   // most 4 * (requests ever queued) + 16 * instances
   h->arena_per_warp = 4 * (int64_t)h->max_nc + 16 * HX_MAX_INST;
+  if (opt && opt->arena_entries > 0) h->arena_per_warp = opt->arena_entries;
   h->chains_per_warp = align_up(std::max(h->max_nq, 1), 256);
   h->topk_per_warp = align_up(h->max_kcap, 32);
   const int64_t w = h->resident_warps;

@@ -71,7 +71,7 @@ class hx_options(ctypes.Structure):
     _fields_ = [("n_record", ctypes.c_int32), ("record_sims", ctypes.c_void_p),
                 ("max_resident_warps", ctypes.c_int32), ("timing", ctypes.c_int32),
                 ("force_generic", ctypes.c_int32), ("n_subset", ctypes.c_int32), ("sim_subset", ctypes.c_void_p),
-                ("checked", ctypes.c_int32)]
+                ("checked", ctypes.c_int32), ("arena_entries", ctypes.c_int32)]
 
 
 class hx_best(ctypes.Structure):
@@ -231,10 +231,11 @@ class Sim:
 
     def __init__(self, traces, cluster, grid, record_sims: Sequence[int] = (), timing: bool = False,
                  max_resident_warps: int = 0, force_generic: bool = False, subset: Optional[Sequence[int]] = None,
-                 checked: bool = False):
+                 checked: bool = False, arena_entries: int = 0):
         """`subset`: run only these simulations (index trace * P + point); the
         others report HX_SKIPPED.  `checked`: also check the scheduler's
-        invariants after every event (per-sim status HX_ERR_INVARIANT)."""
+        invariants after every event (per-sim status HX_ERR_INVARIANT).
+        `arena_entries` (testing) caps each warp's local-queue arena."""
         self.lib = load()
         self.n_traces = len(traces)
         self.n_points = int(grid.alpha_fp.shape[0])
@@ -248,7 +249,8 @@ class Sim:
         self.subset = None if subset is None else [int(s) for s in subset]
         ss = _c(self.subset if self.subset else [0], np.int32)
         opt = hx_options(len(self.record_sims), _p(rs), int(max_resident_warps), int(bool(timing)),
-                         int(bool(force_generic)), len(self.subset or []), _p(ss), int(bool(checked)))
+                         int(bool(force_generic)), len(self.subset or []), _p(ss), int(bool(checked)),
+                         int(arena_entries))
         h = ctypes.c_void_p()
         _check(self.lib, self.lib.hx_sim_create(tr.arr, self.n_traces, ctypes.byref(hc), ctypes.byref(hg),
                                                 ctypes.byref(opt), ctypes.byref(h)))

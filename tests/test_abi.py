@@ -43,7 +43,7 @@ int main(void) {
   S(hx_extra) F(hx_extra, n_done) F(hx_extra, reissued)
   S(hx_grid) F(hx_grid, alpha_fp) F(hx_grid, dispatch_policy)
   S(hx_options) F(hx_options, record_sims) F(hx_options, timing) F(hx_options, force_generic)
-  F(hx_options, n_subset) F(hx_options, sim_subset) F(hx_options, checked)
+  F(hx_options, n_subset) F(hx_options, sim_subset) F(hx_options, checked) F(hx_options, arena_entries)
   S(hx_result) F(hx_result, digest) F(hx_result, status) F(hx_result, cycles_k)
   S(hx_best) F(hx_best, global_sum_p95) F(hx_best, per_trace_point)
   S(hx_info) F(hx_info, resident_warps) F(hx_info, smem_per_block) F(hx_info, generic_kernel)
@@ -161,17 +161,18 @@ def test_rejects_malformed_inputs_without_device_work(lib):
 def test_rejects_bad_subset_and_checked_flag(lib):
     wl = W.make_workload(0, n_queries=20)  # 1 trace x 16 points
 
-    def opt(subset=None, n=None, checked=0):
+    def opt(subset=None, n=None, checked=0, arena=0):
         arr = np.asarray(subset if subset else [0], np.int32)
         o = H.hx_options(0, None, 0, 0, 0, len(subset or []) if n is None else n,
-                         None if subset is None else H._p(arr), checked)
+                         None if subset is None else H._p(arr), checked, arena)
         return o, arr
     for name, (o, keep), msg in [("out of range", opt([3, 16]), "out of range"),
                                  ("negative index", opt([-1]), "out of range"),
                                  ("twice", opt([5, 2, 5]), "twice"),
                                  ("negative count", opt([1], n=-1), "n_subset"),
                                  ("NULL subset", opt(None, n=2), "NULL"),
-                                 ("checked = 2", opt(None, n=0, checked=2), "checked")]:
+                                 ("checked = 2", opt(None, n=0, checked=2), "checked"),
+                                 ("negative arena", opt(None, n=0, arena=-1), "arena_entries")]:
         rc, err, h = _create(lib, wl.traces, wl.cluster, wl.grid, o)
         assert rc == H.HX_ERR_INVALID, name
         assert msg in err, (name, err)

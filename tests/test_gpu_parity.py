@@ -570,3 +570,93 @@ def test_checked_mode_changes_nothing(name, nt, nq):
     o = oracle_results(wl, range(wl.n_sims))
     assert_same(sim.results(), o, f"checked {name}")
     sim.close()
+
+
+def _arena_need(log, n_inst):
+    """Lower and upper bounds of the arena entries one simulation takes: per
+    instance the heap of its largest queue, grown by doubling from 16 (16 +
+    32 + ...); the lower bound counts requests strictly waiting after an
+    event, the upper one also those queued and started in the same event."""
+    def alloc(s):
+        c = tot = 16 if s else 0
+        while s and c < s:
+            c *= 2
+            tot += c
+        return tot
+    lo = hi = 0
+    for m in range(n_inst):
+        sel = log["inst"] == m
+        enq, st = log["enq"][sel], log["start"][sel]
+        cur = top = 0
+        for _, _, d in sorted([(e, 0, 1) for e in enq] + [(s, 1, -1) for s in st]):
+            cur += d
+            top = max(top, cur)
+        hi += alloc(top)
+        w = st > enq
+        cur = top = 0
+        for _, _, d in sorted([(e, 1, 1) for e in enq[w]] + [(s, 0, -1) for s in st[w]]):
+            cur += d
+            top = max(top, cur)
+        lo += alloc(top)
+    return lo, hi
+
+
+@pytest.mark.parametrize("generic", [False, True])
+def test_small_arena_reports_capacity(generic):
+    """A local-queue arena too small for the alpha = 1 queues: those
+    simulations stop with HX_ERR_CAPACITY (no truncation, no fault), the others
+    still match the oracle."""
+    wl = W.make_workload(4, n_traces=1, n_queries=1500)
+    pts = list(range(0, 1024, 64)) + list(range(1024 - 128, 1024, 16))
+    wl = W.Workload(wl.name, wl.traces, wl.cluster, W.subset_grid(wl.grid, pts), wl.objective)
+    arena = 1024
+    sim = gpu(wl, arena_entries=arena, force_generic=generic)
+    r = sim.results()
+    o = oracle_results(wl, range(wl.n_sims))
+    n_cap = n_ok = 0
+    for p in range(wl.n_sims):
+        _, log = oracle.simulate(wl.traces[0], wl.cluster, oracle.point_of(wl.grid, p), log=True)
+        lo, hi = _arena_need(log, wl.cluster.n_inst)
+        if hi <= arena:
+            n_ok += 1
+            assert r["status"][p] == H.HX_OK, p
+        if lo > arena:
+            n_cap += 1
+            assert r["status"][p] == H.HX_ERR_CAPACITY and r["p95_us"][p] == -1, p
+        if r["status"][p] == H.HX_OK:
+            assert_same(r[p:p + 1], o[p:p + 1], f"point {p}")
+        else:
+            assert r["status"][p] == H.HX_ERR_CAPACITY
+    assert n_cap >= 4 and n_ok >= 8
+    sim.close()
+
+
+def test_step_limit_on_endless_reissues():
+    """One instance stopped with a timeout of 1x: every attempt fails after
+    its 2 ms estimate and goes out again to the same instance.  A 20 ms
+    window (10 re-issues) matches the oracle; a 100 s window needs 50000
+    re-issues, more events than the bound (n_calls + n_queries + 8 +
+    16 n_calls + 4096), so the simulation stops with HX_ERR_STEP_LIMIT."""
+    g = cases.load_golden("hand_cases.json")
+    tr = cases.trace_from(g["traces"]["T10_one_query"])
+    pt = dict(alpha_fp=W.SCALE // 2, gamma_fp=W.SCALE, beta_us2=9_000_000, rho=0, local_policy=0, dispatch_policy=0)
+
+    def workload(t1):
+        f = np.zeros(1, W.FAULT_DTYPE)
+        f[0] = (0, 0, 0, t1, 0)
+        cl = W.Cluster(np.array([1000], np.int32), np.array([1000], np.int32), np.array([1], np.int32),
+                       np.zeros(1, np.uint8), 0, 3 * W.SCALE, 0, np.ones(4, np.int32), np.ones(4, np.int32),
+                       None, W.SCALE, f)
+        return W.Workload("stopped", [tr], cl, cases.grid_from_points([pt]), W.OBJ_P95)
+    short = workload(20_000)
+    s = gpu(short)
+    o, oe = oracle.run(short, [0], extra=True)
+    assert int(oe["reissued"][0]) == 10
+    assert_same(s.results(), o, "20 ms window")
+    assert_extras(s.extras(), oe, "20 ms window")
+    s.close()
+    long_ = workload(100_000_000)
+    s = gpu(long_)
+    r = s.results()[0]
+    assert r["status"] == H.HX_ERR_STEP_LIMIT and r["p95_us"] == -1
+    s.close()
