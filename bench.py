@@ -196,10 +196,14 @@ def cpu_baseline(wl, budget_s: float = 20.0):
         if extra:
             n2, e2, dt2, _ = oracle_sample(wl, extra, 8, procs)
             n, events, dt = n + n2, events + e2, dt + dt2
+    # one core, for the per-core rate
+    n1, e1, dt1, _ = oracle_sample(wl, 2, 9, 1)
     return {"value": n / dt, "unit": UNIT, "cores": procs, "kind": "oracle",
             "events_per_s": events / dt,
             "sample": f"{n} seeded random simulations of {wl.name}, one per process, {procs} processes, "
-                      f"{dt:.1f} s wall"}
+                      f"{dt:.1f} s wall",
+            "single_core": {"value": n1 / dt1, "events_per_s": e1 / dt1,
+                            "sample": f"{n1} seeded random simulations in one process, {dt1:.1f} s"}}
 
 
 def run_reference(args):

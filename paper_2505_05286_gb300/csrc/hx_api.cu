@@ -2,6 +2,7 @@
 // the traces into device arrays, per-warp scratch sizing and the launches of
 // the preparation, simulation and best-point kernels on the caller's stream.
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <cstdio>
@@ -17,6 +18,15 @@
 namespace {
 
 thread_local std::string g_err;
+
+// NVTX range over one ABI call (host side: validation, copies, launches), for
+// profilers that group kernels by range (e.g. ncu --nvtx).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 int fail(int code, const std::string& msg) {
   g_err = msg;
@@ -387,6 +397,7 @@ const char* hx_last_error(void) { return g_err.c_str(); }
 
 int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cluster, const hx_grid* grid,
                   const hx_options* opt, hx_sim** out) {
+  NvtxRange range("hx_sim_create");
   if (!out) return fail(HX_ERR_INVALID, "out is NULL");
   *out = nullptr;
   g_err.clear();
@@ -541,6 +552,7 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
 }
 
 int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream) {
+  NvtxRange range("hx_sim_upload");
   if (!h || !traces) return fail(HX_ERR_INVALID, "NULL argument");
   if (n_traces != h->n_traces) return fail(HX_ERR_INVALID, "trace count differs from the handle's");
   for (int t = 0; t < n_traces; ++t)
@@ -567,6 +579,7 @@ int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* str
 }
 
 int hx_sim_run(hx_sim* h, void* stream) {
+  NvtxRange range("hx_sim_run");
   if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   hx::PrepArgs pa;
@@ -654,6 +667,7 @@ int hx_sim_run(hx_sim* h, void* stream) {
 }
 
 int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n) {
+  NvtxRange range("hx_sim_results");
   if (!h || !host_out) return fail(HX_ERR_INVALID, "NULL argument");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
   if ((int64_t)n > h->n_sims) return fail(HX_ERR_INVALID, "n exceeds the number of simulations");
