@@ -37,7 +37,7 @@ def tune(args) -> int:
     cl = W.make_cluster(r)
     tuner = T.OnlineTuner(cl, backend=T.gpu_backend, window_us=int(args.window_s * 1e6), min_queries=5,
                           beta_us2=r.c_ref_us ** 2)
-    T.gpu_backend(T.slice_queries(tr, 0, min(tr.n_queries, 8)), cl, tuner._grid([0]))  # load + first-use costs
+    T.gpu_backend(T.slice_queries(tr, 0, min(tr.n_queries, 8)), cl, tuner.grid_of([0]))  # load + first-use costs
     reps = tuner.run(tr)
     # --time-sweeps: the wall time of a sweep on every window, triggered or
     # not, over the alpha values and over the recipe's whole grid
@@ -47,7 +47,7 @@ def tune(args) -> int:
         for i0, i1 in T.windows(tr, tuner.window_us, tuner.min_queries):
             win = T.slice_queries(tr, i0, i1)
             t0 = time.perf_counter()
-            T.gpu_backend(win, cl, tuner._grid(tuner.alphas))
+            T.gpu_backend(win, cl, tuner.grid_of(tuner.alphas))
             sweep_ms.append(1000 * (time.perf_counter() - t0))
             t0 = time.perf_counter()
             sim = H.Sim([win], cl, full)

@@ -122,7 +122,8 @@ class OnlineTuner:
         self.min_queries = min_queries
         self.p_threshold = p_threshold
 
-    def _grid(self, alphas: Sequence[int]) -> W.Grid:
+    def grid_of(self, alphas: Sequence[int]) -> W.Grid:
+        """Grid of the given alpha values with this tuner's gamma, rho and beta."""
         n = len(alphas)
         return W.Grid(np.asarray(alphas, np.int64), np.full(n, self.gamma_fp, np.int64),
                       np.full(n, self.rho, np.int32), np.full(n, self.beta, np.int64),
@@ -134,14 +135,14 @@ class OnlineTuner:
         ref_lat = None
         for w, (i0, i1) in enumerate(windows(trace, self.window_us, self.min_queries)):
             win = slice_queries(trace, i0, i1)
-            _, lat = self.backend(win, self.cluster, self._grid([alpha]))
+            _, lat = self.backend(win, self.cluster, self.grid_of([alpha]))
             p = welch_greater(lat, ref_lat) if ref_lat is not None else None
             trig = p is not None and p < self.p_threshold
             rep = WindowReport(w, int(trace.arrival_us[i0]), int(trace.arrival_us[i1 - 1]), i1 - i0, alpha,
                                nearest_rank_p95(lat), p, trig, alpha)
             if trig:
                 t0 = time.perf_counter()
-                res, _ = self.backend(win, self.cluster, self._grid(self.alphas))
+                res, _ = self.backend(win, self.cluster, self.grid_of(self.alphas))
                 p95 = res["p95_us"].astype(np.int64)
                 ok = res["status"] == 0
                 best = int(np.argmin(np.where(ok, p95, np.iinfo(np.int64).max)))  # ties: lowest alpha

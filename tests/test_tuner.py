@@ -25,7 +25,7 @@ def test_slice_is_a_valid_trace():
     tr, cl, _ = C.shift_scenario()
     win = T.slice_queries(tr, 100, 140)
     assert win.arrival_us[0] == 0 and win.call_base[0] == 0 and win.call_base[-1] == win.n_calls
-    res, lat = C.oracle_backend(win, cl, T.OnlineTuner(cl)._grid([0]))
+    res, lat = C.oracle_backend(win, cl, T.OnlineTuner(cl).grid_of([0]))
     assert res["status"][0] == 0 and len(lat) == 40 and (lat > 0).all()
 
 
