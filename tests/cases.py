@@ -78,9 +78,11 @@ def uniform_single_instance(n, arrivals, svc_us=1000, slots=1):
     return tr, cl
 
 
-def random_workload(seed):
+def random_workload(seed, lean=False):
     """A small random but valid workload: any cluster shape, k from 0 to 8,
-    retries up to R, tenants, fault windows, mixed policies."""
+    retries up to R, tenants, fault windows, mixed policies.  `lean` keeps
+    the shapes but drops tenants and fault windows and puts every point on
+    WB + the urgency queue (the domain of the benchmark's kernel)."""
     rng = np.random.default_rng(1000 + seed)
     T = int(rng.integers(1, 5))
     N = int(rng.integers(1, 65))
@@ -131,4 +133,12 @@ def random_workload(seed):
                   rng.integers(0, 4, P).astype(np.int32), rng.integers(0, 10 ** 12, P).astype(np.int64),
                   rng.integers(0, 3, P).astype(np.uint8), rng.integers(0, 2, P).astype(np.uint8))
     grid.alpha_fp[0], grid.alpha_fp[1] = 0, W.SCALE
-    return W.Workload(f"random {seed}", [tr], cl, grid, int(rng.integers(0, 2)))
+    objective = int(rng.integers(0, 2))
+    if lean:
+        cl = W.Cluster(cl.prefill_tok_s, cl.decode_us_tok, cl.slots, cl.inst_type, cl.ref_type, cl.slo_mult_fp,
+                       cl.rmax, cl.stage_ref_prompt, cl.stage_ref_out)
+        tr.tenant = None
+        grid.local_policy[:] = W.POLICY_PQ
+        grid.dispatch_policy[:] = W.DISPATCH_WB
+        return W.Workload(f"random lean {seed}", [tr], cl, grid, objective)
+    return W.Workload(f"random {seed}", [tr], cl, grid, objective)

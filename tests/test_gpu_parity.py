@@ -519,6 +519,21 @@ def test_random_small_workloads(seed):
     sim.close()
 
 
+@pytest.mark.parametrize("seed", range(24))
+def test_random_small_workloads_lean(seed):
+    """The same random shapes (any instance count and slots, k from 0 to 8)
+    on WB + the urgency queue alone, so that the benchmark's lean kernel runs
+    them: every simulation and the best points equal the oracle's."""
+    wl = cases.random_workload(seed, lean=True)
+    sim = gpu(wl)
+    assert sim.info()["generic_kernel"] == 0
+    o = oracle_results(wl, range(wl.n_sims))
+    assert (o["status"] == 0).all()
+    assert_same(sim.results(), o, wl.name)
+    check_best(sim, wl, o)
+    sim.close()
+
+
 def test_command_line(capsys):
     import json
     from paper_2505_05286_gb300 import __main__ as cli

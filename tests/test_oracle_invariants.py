@@ -274,12 +274,14 @@ def test_faulty_recipe_reissues(dispatch):
     assert total > 0
 
 
+@pytest.mark.parametrize("lean", [False, True])
 @pytest.mark.parametrize("seed", range(24))
-def test_invariants_random_workloads(seed):
+def test_invariants_random_workloads(seed, lean):
     """Random clusters, traces (k from 0 to 8), tenants, fault windows and
-    mixed policies: the schedule invariants and the per-tenant counts hold."""
+    mixed policies (or, lean, the same shapes on WB + urgency queue alone):
+    the schedule invariants and the per-tenant counts hold."""
     from tests import cases
-    wl = cases.random_workload(seed)
+    wl = cases.random_workload(seed, lean)
     tr = wl.traces[0]
     p = oracle.prep(tr, wl.cluster)
     for pt_i in range(wl.grid.n_points):
