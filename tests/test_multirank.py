@@ -5,7 +5,6 @@ import os
 import socket
 
 import numpy as np
-import pytest
 
 import oracle
 from paper_2505_05286_gb300 import dist as D

@@ -1,6 +1,5 @@
 """Host-side per-tenant views: Jain's fairness index and per-tenant P95,
 pinned by closed forms and the hand-worked two-tenant schedule."""
-import numpy as np
 import pytest
 
 import oracle

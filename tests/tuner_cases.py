@@ -1,5 +1,4 @@
 """Shared pieces of the online-tuning tests."""
-import numpy as np
 
 import oracle
 from paper_2505_05286_gb300 import tuner as T
