@@ -408,7 +408,16 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   if ((rc = validate_grid(grid))) return rc;
   for (int t = 0; t < n_traces; ++t)
     if ((rc = validate_trace(&traces[t], t, cluster, min_prefill, max_decode))) return rc;
-  if (opt && opt->n_record > 0 && !opt->record_sims) return fail(HX_ERR_INVALID, "record_sims is NULL");
+  if (opt && opt->n_record < 0) return fail(HX_ERR_INVALID, "n_record < 0");
+  if (opt && opt->n_record > 0) {
+    if (!opt->record_sims) return fail(HX_ERR_INVALID, "record_sims is NULL");
+    std::vector<int32_t> sorted(opt->record_sims, opt->record_sims + opt->n_record);
+    std::sort(sorted.begin(), sorted.end());
+    const int64_t n_sims = (int64_t)n_traces * grid->n_points;
+    for (size_t j = 0; j < sorted.size(); ++j)
+      if (sorted[j] < 0 || sorted[j] >= n_sims || (j > 0 && sorted[j] == sorted[j - 1]))
+        return fail(HX_ERR_INVALID, "record_sims must be distinct valid sim indices");
+  }
   if (opt && opt->checked != 0 && opt->checked != 1) return fail(HX_ERR_INVALID, "checked must be 0 or 1");
   if (opt && opt->arena_entries < 0) return fail(HX_ERR_INVALID, "arena_entries < 0");
   std::vector<int64_t> subset;
@@ -527,9 +536,7 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
     h->rec_stride = std::max(h->max_nc, 1);
     std::vector<int32_t> map((size_t)h->n_sims, -1);
     for (int j = 0; j < opt->n_record; ++j) {
-      const int32_t sim = opt->record_sims[j];
-      if (sim < 0 || sim >= h->n_sims || map[sim] >= 0)
-        return bail(fail(HX_ERR_INVALID, "record_sims must be distinct valid sim indices"));
+      const int32_t sim = opt->record_sims[j];  // checked above: distinct, in range
       map[sim] = j;
       h->record_sims.push_back(sim);
     }

@@ -158,21 +158,27 @@ def test_rejects_malformed_inputs_without_device_work(lib):
         assert not h.value
 
 
-def test_rejects_bad_subset_and_checked_flag(lib):
+def test_rejects_bad_options(lib):
     wl = W.make_workload(0, n_queries=20)  # 1 trace x 16 points
 
-    def opt(subset=None, n=None, checked=0, arena=0):
+    def opt(subset=None, n=None, checked=0, arena=0, record=None, n_record=None):
         arr = np.asarray(subset if subset else [0], np.int32)
-        o = H.hx_options(0, None, 0, 0, 0, len(subset or []) if n is None else n,
+        rec = np.asarray(record if record else [0], np.int32)
+        o = H.hx_options(len(record or []) if n_record is None else n_record,
+                         None if record is None else H._p(rec), 0, 0, 0,
+                         len(subset or []) if n is None else n,
                          None if subset is None else H._p(arr), checked, arena)
-        return o, arr
+        return o, (arr, rec)
     for name, (o, keep), msg in [("out of range", opt([3, 16]), "out of range"),
                                  ("negative index", opt([-1]), "out of range"),
                                  ("twice", opt([5, 2, 5]), "twice"),
                                  ("negative count", opt([1], n=-1), "n_subset"),
                                  ("NULL subset", opt(None, n=2), "NULL"),
                                  ("checked = 2", opt(None, n=0, checked=2), "checked"),
-                                 ("negative arena", opt(None, n=0, arena=-1), "arena_entries")]:
+                                 ("negative arena", opt(None, n=0, arena=-1), "arena_entries"),
+                                 ("record out of range", opt(None, n=0, record=[16]), "record_sims"),
+                                 ("record twice", opt(None, n=0, record=[3, 3]), "record_sims"),
+                                 ("negative n_record", opt(None, n=0, n_record=-1), "n_record")]:
         rc, err, h = _create(lib, wl.traces, wl.cluster, wl.grid, o)
         assert rc == H.HX_ERR_INVALID, name
         assert msg in err, (name, err)
