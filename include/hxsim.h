@@ -159,8 +159,9 @@ typedef struct hx_grid {
 } hx_grid;
 
 typedef struct hx_options {
-  int32_t n_record;                 /* simulations whose per-call log is kept */
-  const int32_t* record_sims;       /* [n_record] sim indices (trace * P + point) */
+  int32_t n_record;                 /* >= 0 simulations whose per-call log is kept (runs
+                                       the generic kernel) */
+  const int32_t* record_sims;       /* [n_record] distinct sim indices (trace * P + point) */
   int32_t max_resident_warps;       /* 0 = fill the GPU */
   int32_t timing;                   /* 1 = time each kernel with CUDA events */
   int32_t force_generic;            /* 1 = always use the simulation kernel built for
