@@ -97,11 +97,19 @@ static int64_t stage_ref(const hxo_cluster* cl, int s) {
   return sum / cl->n_inst;
 }
 
-/* Digest term of a (time, id << 8 | tag) pair:
- * y = ((time * 0x9E3779B97F4A7C15) xor idtag) * 0xBF58476D1CE4E5B9, term = y xor (y >> 32). */
+/* The splitmix64 output function (Steele, Lea & Flood, "Fast splittable
+ * pseudorandom number generators", OOPSLA 2014): two xor-shift-multiply
+ * rounds and a final xor-shift, each a bijection of 64-bit words. */
+static uint64_t splitmix64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+  return z ^ (z >> 31);
+}
+
+/* Digest term of a (time, id << 8 | tag) pair: the splitmix64 output
+ * function of (time * 0x9E3779B97F4A7C15) xor idtag. */
 static uint64_t digest_term(uint64_t t, uint64_t idtag) {
-  uint64_t y = ((t * 0x9E3779B97F4A7C15ULL) ^ idtag) * 0xBF58476D1CE4E5B9ULL;
-  return y ^ (y >> 32);
+  return splitmix64_mix((t * 0x9E3779B97F4A7C15ULL) ^ idtag);
 }
 
 static uint64_t call_term(int32_t rid, int inst, int64_t start) {

@@ -14,15 +14,19 @@ namespace hx {
 // ------------------------------------------------------------------ helpers
 __device__ __forceinline__ int64_t ceil_div_pos(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-constexpr uint64_t kDigestMul = 0x9E3779B97F4A7C15ull;
-constexpr uint64_t kDigestMix = 0xBF58476D1CE4E5B9ull;
+constexpr uint64_t kDigestMul = 0x9E3779B97F4A7C15ull;  // golden-ratio increment of splitmix64
+constexpr uint64_t kMixA = 0xBF58476D1CE4E5B9ull;       // splitmix64 output-function multipliers
+constexpr uint64_t kMixB = 0x94D049BB133111EBull;       // (Steele, Lea & Flood, OOPSLA 2014)
 
-// Digest terms: y = ((time * phi) xor (id << 8 | tag)) * c, term = y xor (y >> 32);
-// each step is a bijection, so a change of any one call's instance or start
-// (or any query's end) changes the sum.
+// Digest terms: the splitmix64 output function (two xor-shift-multiply rounds
+// and a final xor-shift) of (time * phi) xor (id << 8 | tag); every step is a
+// bijection, so a change of any one call's instance or start (or any query's
+// end) changes the sum.
 __device__ __forceinline__ uint64_t digest_term(uint64_t t, uint64_t idtag) {
-  const uint64_t y = ((t * kDigestMul) ^ idtag) * kDigestMix;
-  return y ^ (y >> 32);
+  uint64_t z = (t * kDigestMul) ^ idtag;
+  z = (z ^ (z >> 30)) * kMixA;
+  z = (z ^ (z >> 27)) * kMixB;
+  return z ^ (z >> 31);
 }
 
 // Id tags: a call's start is (rid << 8 | instance), a query's end (qid << 8 | 0xFF).

@@ -36,6 +36,8 @@ def _release_times(tr, end):
 
 
 def _mix64(z):
+    """The splitmix64 output function (Steele, Lea & Flood 2014), in Python
+    integers, for the digest recomputed from a log."""
     m = (1 << 64) - 1
     z &= m
     z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & m
@@ -98,11 +100,10 @@ def check_schedule(tr, cl, res, log, reissued=0):
         assert int(res["makespan_us"]) == int(end.max())
     if reissued:
         return
-    gold, mixc, m64 = 0x9E3779B97F4A7C15, 0xBF58476D1CE4E5B9, (1 << 64) - 1
+    gold, m64 = 0x9E3779B97F4A7C15, (1 << 64) - 1
 
     def term(t, idtag):
-        y = ((((t * gold) & m64) ^ idtag) * mixc) & m64
-        return y ^ (y >> 32)
+        return _mix64(((t * gold) & m64) ^ idtag)
 
     dig = 0
     for c in range(tr.n_calls):
