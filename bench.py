@@ -173,37 +173,95 @@ def _barrier(world):
         dist.barrier()
 
 
-def oracle_sample(wl, n_sims: int, seed: int, procs: int):
-    """Seeded sample of simulations of `wl` run by the CPU oracle."""
+# ------------------------------------------------------------------ oracle
+# The CPU oracle as it stands, one simulation per job in a pool of worker
+# processes (spawn), each job timing its own simulation on its core.  A
+# worker builds only the traces its jobs need (one-trace workloads of the
+# same recipe, same cut and same grid).
+_ORACLE_ARGS = None
+_ORACLE_CACHE = {}
+
+
+def _oracle_init(args_dict):
+    global _ORACLE_ARGS
     import oracle
+    oracle.build()
+    _ORACLE_ARGS = argparse.Namespace(**args_dict)
+
+
+def _oracle_one(sim_trace_point):
+    import oracle
+    sim, t, p = sim_trace_point
+    if t not in _ORACLE_CACHE:
+        if len(_ORACLE_CACHE) >= 8:
+            _ORACLE_CACHE.pop(next(iter(_ORACLE_CACHE)))
+        a = argparse.Namespace(**vars(_ORACLE_ARGS))
+        a.traces = 1
+        _ORACLE_CACHE[t] = _workload(a, first_trace=t)
+    wl = _ORACLE_CACHE[t]
+    w0 = time.time()
+    c0 = time.perf_counter()
+    r = oracle.simulate(wl.traces[0], wl.cluster, oracle.point_of(wl.grid, p))
+    return sim, time.perf_counter() - c0, w0, time.time(), int(r["events"]), int(r["status"])
+
+
+def stratified_sims(wl, n: int, seed: int):
+    """n simulations drawn evenly over the grid's alpha values (trace and the
+    other axes at random, no repeats), or every simulation if n >= n_sims.
+    Every recipe's grid gives each alpha value the same number of points, so
+    an even draw per alpha value is proportional to the workload."""
+    if n >= wl.n_sims:
+        return list(range(wl.n_sims))
+    g = wl.grid
+    P, T = g.n_points, len(wl.traces)
+    vals = np.unique(g.alpha_fp)
     rng = np.random.default_rng(seed)
-    sims = sorted(rng.choice(wl.n_sims, size=min(n_sims, wl.n_sims), replace=False).tolist())
-    t0 = time.perf_counter()
-    oracle.run(wl, sims, procs=procs)
-    dt = time.perf_counter() - t0
+    sims = []
+    for i, a in enumerate(vals):
+        pts = np.nonzero(g.alpha_fp == a)[0]
+        k = n // len(vals) + (1 if i < n % len(vals) else 0)
+        pick = rng.choice(T * pts.size, size=min(k, T * pts.size), replace=False)
+        sims += (pick // pts.size * P + pts[pick % pts.size]).tolist()
+    return sorted(sims)
+
+
+def oracle_timed(args, wl, sims, procs: int, first_trace: int = 0):
+    """Run the listed simulations of `wl` with the oracle; returns the number
+    run, their completed calls, the sum of the per-simulation times (one
+    core each) and the wall time from the first start to the last end."""
+    import multiprocessing as mp
     P = wl.grid.n_points
-    events = sum(wl.traces[s // P].n_calls for s in sims)
-    return len(sims), events, dt, sims
+    jobs = [(s, first_trace + s // P, s % P) for s in sims]
+    jobs.sort(key=lambda j: j[1])  # neighbours share a trace in the workers' caches
+    spec = {k: v for k, v in vars(args).items()}
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(procs, initializer=_oracle_init, initargs=(spec,)) as pool:
+        out = pool.map(_oracle_one, jobs, chunksize=1)
+    if any(o[5] != 0 for o in out):
+        raise RuntimeError("the oracle reported a failed simulation")
+    core_s = sum(o[1] for o in out)
+    wall = max(o[3] for o in out) - min(o[2] for o in out)
+    return len(out), sum(o[4] for o in out), core_s, wall
 
 
-def cpu_baseline(wl, budget_s: float = 20.0):
+def cpu_baseline(args, wl, n_sample: int):
+    """The oracle on the host's cores: every simulation of the workload when
+    n_sample >= n_sims, else n_sample drawn evenly over the alpha values.
+    The single-core rate is the sample over the sum of its per-simulation
+    times (each ran alone on one core); the all-core rate is the sample over
+    the wall time of the pool."""
     procs = os.cpu_count() or 1
-    n, events, dt, _ = oracle_sample(wl, max(procs, 16), 7, procs)
-    # scale the sample toward the time budget once
-    if dt < budget_s / 3:
-        extra = int(n * (budget_s / max(dt, 1e-3) - 1))
-        extra = max(0, min(extra, 4 * procs * 4))
-        if extra:
-            n2, e2, dt2, _ = oracle_sample(wl, extra, 8, procs)
-            n, events, dt = n + n2, events + e2, dt + dt2
-    # one core, for the per-core rate
-    n1, e1, dt1, _ = oracle_sample(wl, 2, 9, 1)
-    return {"value": n / dt, "unit": UNIT, "cores": procs, "kind": "oracle",
-            "events_per_s": events / dt,
-            "sample": f"{n} seeded random simulations of {wl.name}, one per process, {procs} processes, "
-                      f"{dt:.1f} s wall",
-            "single_core": {"value": n1 / dt1, "events_per_s": e1 / dt1,
-                            "sample": f"{n1} seeded random simulations in one process, {dt1:.1f} s"}}
+    sims = stratified_sims(wl, n_sample, 7)
+    n, events, core_s, wall = oracle_timed(args, wl, sims, procs)
+    whole = n == wl.n_sims
+    what = (f"every simulation of {wl.name}" if whole else
+            f"{n} of the {wl.n_sims} simulations of {wl.name}, {n // len(np.unique(wl.grid.alpha_fp))} per alpha "
+            f"value (proportional to the grid); rates extrapolate to the whole workload as the sample's mean cost")
+    return {"value": n / wall, "unit": UNIT, "cores": procs, "kind": "oracle", "events_per_s": events / wall,
+            "sample": f"{what}; one simulation per job on {procs} processes, {wall:.1f} s wall",
+            "single_core": {"value": n / core_s, "events_per_s": events / core_s,
+                            "sample": f"the same {n} simulations, sum of their one-core times {core_s:.1f} s"},
+            "sims": n, "whole_workload": whole}
 
 
 def run_reference(args):
@@ -214,11 +272,11 @@ def run_reference(args):
     procs = os.cpu_count() or 1
     per_step = max(procs, 16)
     for w in range(args.warmup):
-        oracle_sample(wl, max(2, procs // 4), 1000 + w, procs)
+        oracle_timed(args, wl, stratified_sims(wl, max(2, procs // 4), 1000 + w), procs)
     t = 0.0
     n_tot = ev_tot = 0
     for k in range(args.steps):
-        n, ev, dt, _ = oracle_sample(wl, per_step, 2000 + k, procs)
+        n, ev, _, dt = oracle_timed(args, wl, stratified_sims(wl, per_step, 2000 + k), procs)
         t += dt
         n_tot += n
         ev_tot += ev
@@ -230,7 +288,8 @@ def run_reference(args):
             "config": {"workload": wl.name, "sims": wl.n_sims, "sample_sims_per_step": per_step,
                        "l2": "oracle on host cores"},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": procs, "kind": "oracle",
-                             "sample": f"{per_step} seeded random simulations per step, one per process"},
+                             "sample": f"{per_step} simulations per step drawn evenly over the alpha values, "
+                                       f"one per job on {procs} processes"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -262,7 +321,6 @@ def run_gpu(args):
     torch.cuda.synchronize()
 
     # kernel-only timing: inputs resident, K steps between events on the stream
-    sim_ms = []
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     _barrier(world)
     torch.cuda.synchronize()
@@ -274,8 +332,8 @@ def run_gpu(args):
         torch.cuda.synchronize()
     _barrier(world)
     t_ms = start.elapsed_time(stop)
-    # per-kernel times of the last timed step (events the library records on the same stream)
-    sim_ms.append(sim.timings())
+    # per-kernel times of every timed step (events the library records on the same stream)
+    sim_ms = [sim.timings(back) for back in range(min(args.steps, 64))]
     t_ms = D.max_over_ranks(t_ms)
     res = sim.results()
     ok = bool((res["status"] == 0).all())
@@ -356,7 +414,8 @@ def run_gpu(args):
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                     "steps": e2e_steps}}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl)
+        n_sample = args.cpu_sample if args.cpu_sample else (wl.n_sims if wl.n_sims <= 8192 else 256)
+        line["cpu_baseline"] = cpu_baseline(args, wl, n_sample)
     if rank == 0:
         print(json.dumps(line), flush=True)
     sim.close()
@@ -372,6 +431,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample", type=int, default=0,
+                    help="simulations the oracle runs for cpu_baseline (default: every one up to 8192, else 256 "
+                         "drawn evenly over the alpha values)")
     ap.add_argument("--traces", type=int, default=None, help="cut the workload to this many traces (profiling)")
     ap.add_argument("--queries", type=int, default=None, help="cut each trace to this many queries (profiling)")
     ap.add_argument("--alpha", default="all", choices=["all", "1", "lt1"],

@@ -215,7 +215,16 @@ typedef struct hx_extra {
 typedef struct hx_sim hx_sim;
 
 /* Validate and copy traces, cluster and grid to library-owned device memory
- * and size the per-warp scratch.  On failure *out is NULL. */
+ * and size the per-warp scratch.  On failure *out is NULL.
+ *
+ * Defines the simulations of Sec. 4.3's alpha tuning: every (trace, point)
+ * pair replays the trace through the scheduler of Sec. 4.1 (Eq. comp for
+ * t_comp, the queue cost t_queue, Eq. score) and Sec. 4.2 (the SLO budget at
+ * send time, Eq. priority), over the workflow of Sec. 2.1 on the instance
+ * profiles of Sec. 3.3.  `traces` [n_traces] and the cluster and grid arrays
+ * are host memory the caller keeps; `opt` may be NULL.  Errors:
+ * HX_ERR_INVALID (input outside the domain above, with a message),
+ * HX_ERR_OOM, HX_ERR_CUDA. */
 int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cluster,
                   const hx_grid* grid, const hx_options* opt, hx_sim** out);
 
@@ -226,18 +235,32 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
 int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream);
 
 /* Enqueue the whole path on `stream` (a cudaStream_t, NULL = legacy default):
- * per-call preparation, every simulation, the best-point reduction.
- * Asynchronous; may be called repeatedly. */
+ * per-call preparation (Eq. comp per call and instance type, the mean cost
+ * tbar of Sec. 4.2, the query deadline of Sec. 5.1's SLO), every
+ * simulation (Sec. 4.1 dispatch and Sec. 4.2 local queues, event by event,
+ * reduced to Sec. 4.3's T_0.95 and the SLO count), and the best-point
+ * reduction (Sec. 4.3's argmin over the grid).  Asynchronous; may be called
+ * repeatedly.  Errors: HX_ERR_INVALID (NULL handle), HX_ERR_CUDA (a launch
+ * failed); per-simulation problems are reported in hx_result.status. */
 int hx_sim_run(hx_sim* h, void* stream);
 
-/* Wait for the last run and copy n <= n_sims results to host memory. */
+/* Wait for the last run and copy n <= n_sims results to host memory
+ * (`host_out` [n], caller-owned): per simulation Sec. 4.3's objective T_0.95
+ * (the nearest-rank P95 of query latency), the number of queries within
+ * their SLO (Sec. 5.1: latency <= slo_mult times the exclusive latency),
+ * makespan, completed calls, the digest and the status.  Errors:
+ * HX_ERR_STATE before a run, HX_ERR_INVALID (n too large), HX_ERR_CUDA. */
 int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n);
 
 /* Wait for the last run and copy n <= n_sims per-tenant counts (see
- * hx_extra); same indexing as hx_sim_results. */
+ * hx_extra; Sec. 5's multi-tenant SLO attainment); same indexing as
+ * hx_sim_results. */
 int hx_sim_extras(hx_sim* h, hx_extra* host_out, size_t n);
 
-/* Wait for the last run and return the best point for `objective`. */
+/* Wait for the last run and return the best point for `objective`:
+ * Sec. 4.3's alpha* = argmin T_0.95 per trace and over the grid (sum over
+ * traces), or the same among points with >= 95% SLO attainment.
+ * out->per_trace_point, if not NULL, is caller memory of n_traces. */
 int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out);
 
 /* Per-point sums over the handle's traces from the last run (the partial
@@ -272,6 +295,11 @@ int hx_sim_prep(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int3
  * opt.timing = 1.  Waits for the run. */
 int hx_sim_timings(hx_sim* h, float* prep_ms, float* sim_ms, float* best_ms);
 
+/* The same for an earlier run: back = 0 is the last run, 1 the one before,
+ * up to min(runs, 64) - 1 (the handle keeps the events of its last 64
+ * runs).  Waits for that run.  HX_ERR_INVALID for `back` out of range. */
+int hx_sim_timings_back(hx_sim* h, int32_t back, float* prep_ms, float* sim_ms, float* best_ms);
+
 /* Size of the device array behind hx_sim_run_static. */
 #define HX_STATIC_SCRATCH_BYTES (64u << 20)
 
@@ -293,11 +321,15 @@ int hx_sim_timings(hx_sim* h, float* prep_ms, float* sim_ms, float* best_ms);
  * bytes it would need.  Fewer warps run when the trace is large, so results
  * are the same as hx_sim_run's but throughput is lower.
  *
- * The first call on a device looks up that device's address of the array
- * (cudaGetSymbolAddress, with that device current); make it before any stream
- * capture.  Runs on `stream` and returns when the results are in `results`.
- * Every call on a device shares the one array: calls that overlap on the GPU
- * (other threads, other streams) race and corrupt each other. */
+ * A call made while `stream` is not capturing looks up the current device's
+ * address of the array (cudaGetSymbolAddress, with that device current), so
+ * a device reset between calls is harmless; a call made during stream
+ * capture reuses the address of the last earlier call on that device, so
+ * the first call on a device must come before any stream capture
+ * (HX_ERR_STATE otherwise).  Runs on `stream` and returns when the results
+ * are in `results`.  Every call on a device shares the one array, whose
+ * contents the next call overwrites: calls that overlap on the GPU (other
+ * threads, other streams) race and corrupt each other. */
 int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluster, const hx_grid* grid,
                       int32_t objective, hx_result* results, hx_best* best, void* stream);
 
@@ -325,7 +357,8 @@ typedef struct hx_info {
 
 int hx_sim_info(hx_sim* h, hx_info* out);
 
-/* Free everything; NULL is allowed. */
+/* Wait for the handle's last run and free everything it holds (the end of
+ * the tuning pass of Sec. 4.3); NULL is allowed.  Always HX_OK. */
 int hx_sim_destroy(hx_sim* h);
 
 /* The calling thread's last error message ("" if none). */

@@ -47,6 +47,45 @@ constexpr int64_t kHorizonMax = int64_t(1) << 39; // last arrival + all service,
 
 int64_t align_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 
+// The dynamic shared-memory limit of a kernel (cudaFuncAttributeMax-
+// DynamicSharedMemorySize) is one setting per function and device, shared by
+// every handle in the process.  It is set, under a mutex, to the largest size
+// any launch of that kernel on that device has asked for, so a later handle
+// or static call with a smaller cluster never lowers it below what an earlier
+// handle launches with.  Called before every launch; it sets the attribute
+// each time (a host-side call), so a device reset cannot leave it lower than
+// the record says.
+constexpr int kMaxDevices = 64;
+std::mutex g_smem_mu;
+int g_smem_limit[kMaxDevices][2] = {};  // [device][0: hx_sim_kernel, 1: hx_sim_kernel_lean]
+
+int ensure_dyn_smem(bool generic, int bytes) {
+  int dev = 0;
+  HX_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return fail(HX_ERR_INVALID, "device index out of range");
+  std::lock_guard<std::mutex> lock(g_smem_mu);
+  int& cur = g_smem_limit[dev][generic ? 0 : 1];
+  const int want = std::max(cur, bytes);
+  const void* kfn = generic ? (const void*)hx::hx_sim_kernel : (const void*)hx::hx_sim_kernel_lean;
+  if (cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, want) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(HX_ERR_CUDA, "cannot reserve " + std::to_string(want) +
+                                 " bytes of shared memory for the simulation kernel");
+  }
+  cur = want;
+  return HX_OK;
+}
+
+// The lean instantiation serves grids that are all workload-balanced dispatch
+// with the urgency queue, log nothing, check nothing, count one tenant and
+// have no fault windows.
+bool needs_generic(const hx_grid* grid, const hx::ClusterK& ck, bool record, bool force, bool checked) {
+  if (record || force || checked || ck.n_tenants > 1 || ck.n_faults > 0) return true;
+  for (int p = 0; p < grid->n_points; ++p)
+    if (grid->local_policy[p] != HX_LOCAL_PQ || grid->dispatch_policy[p] != HX_DISPATCH_WB) return true;
+  return false;
+}
+
 }  // namespace
 
 struct hx_sim {
@@ -110,7 +149,12 @@ struct hx_sim {
   cudaStream_t last_stream = nullptr;
   bool ran = false;
   bool timing = false;
-  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  // with timing: four events per run (before prep, before and after the
+  // simulations, after the best point) for the last kTimedRuns runs
+  static constexpr int kTimedRuns = 64;
+  std::vector<cudaEvent_t> ev;
+  int64_t runs = 0;
+  cudaEvent_t* run_ev(int64_t r) { return ev.data() + 4 * (r % kTimedRuns); }
   std::vector<void*> allocs;
 
   template <class T>
@@ -130,7 +174,7 @@ struct hx_sim {
 
   ~hx_sim() {
     for (void* p : allocs) cudaFree(p);
-    for (auto& e : ev)
+    for (auto e : ev)
       if (e) cudaEventDestroy(e);
   }
 };
@@ -489,20 +533,11 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
                           (rc = upload(h->d_subset, subset.data(), (int64_t)subset.size(), s0))))
     return bail(rc);
 
-  // the lean instantiation serves grids that are all workload-balanced
-  // dispatch with the urgency queue, log nothing, count one tenant and have
-  // no fault windows
-  h->generic = (opt && (opt->n_record > 0 || opt->force_generic)) || h->checked || ck.n_tenants > 1 ||
-               ck.n_faults > 0;
-  for (int p = 0; p < grid->n_points && !h->generic; ++p)
-    if (grid->local_policy[p] != HX_LOCAL_PQ || grid->dispatch_policy[p] != HX_DISPATCH_WB) h->generic = true;
+  h->generic = needs_generic(grid, ck, opt && opt->n_record > 0, opt && opt->force_generic, h->checked);
   const void* kfn = h->generic ? (const void*)hx::hx_sim_kernel : (const void*)hx::hx_sim_kernel_lean;
   // launch shape of the simulation kernel and its per-warp scratch
   h->smem_per_block = hx::kWarpsPerBlock * ck.smem_per_warp;
-  if (cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, h->smem_per_block) != cudaSuccess) {
-    cudaGetLastError();
-    return bail(fail(HX_ERR_CUDA, "cannot reserve shared memory for the simulation kernel"));
-  }
+  if ((rc = ensure_dyn_smem(h->generic, h->smem_per_block))) return bail(rc);
   int bps = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, kfn, hx::kWarpsPerBlock * 32, h->smem_per_block) !=
           cudaSuccess ||
@@ -550,6 +585,7 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   }
   if (opt && opt->timing) {
     h->timing = true;
+    h->ev.assign(4 * hx_sim::kTimedRuns, nullptr);
     for (auto& e : h->ev)
       if (cudaEventCreate(&e) != cudaSuccess) return bail(fail(HX_ERR_CUDA, "cudaEventCreate failed"));
   }
@@ -655,21 +691,24 @@ int hx_sim_run(hx_sim* h, void* stream) {
   ba.point_sums = h->d_point_sums;
 
   const int prep_blocks = (int)std::max<int64_t>(1, (h->n_q + 255) / 256);
-  if (h->timing) HX_CUDA(cudaEventRecord(h->ev[0], s));
+  if (int rc = ensure_dyn_smem(h->generic, h->smem_per_block)) return rc;
+  cudaEvent_t* ev = h->timing ? h->run_ev(h->runs) : nullptr;
+  if (ev) HX_CUDA(cudaEventRecord(ev[0], s));
   hx::hx_prep_kernel<<<prep_blocks, 256, 0, s>>>(pa, h->ck);
   HX_CUDA(cudaGetLastError());
-  if (h->timing) HX_CUDA(cudaEventRecord(h->ev[1], s));
+  if (ev) HX_CUDA(cudaEventRecord(ev[1], s));
   if (h->generic)
     hx::hx_sim_kernel<<<h->blocks, hx::kWarpsPerBlock * 32, h->smem_per_block, s>>>(sa, h->ck);
   else
     hx::hx_sim_kernel_lean<<<h->blocks, hx::kWarpsPerBlock * 32, h->smem_per_block, s>>>(sa, h->ck);
   HX_CUDA(cudaGetLastError());
-  if (h->timing) HX_CUDA(cudaEventRecord(h->ev[2], s));
+  if (ev) HX_CUDA(cudaEventRecord(ev[2], s));
   hx::hx_best_kernel<<<h->n_traces + 1, 256, 0, s>>>(ba);
   HX_CUDA(cudaGetLastError());
-  if (h->timing) HX_CUDA(cudaEventRecord(h->ev[3], s));
+  if (ev) HX_CUDA(cudaEventRecord(ev[3], s));
   h->last_stream = s;
   h->ran = true;
+  h->runs++;
   return HX_OK;
 }
 
@@ -835,14 +874,21 @@ int hx_sim_prep(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int3
 }
 
 int hx_sim_timings(hx_sim* h, float* prep_ms, float* sim_ms, float* best_ms) {
+  return hx_sim_timings_back(h, 0, prep_ms, sim_ms, best_ms);
+}
+
+int hx_sim_timings_back(hx_sim* h, int32_t back, float* prep_ms, float* sim_ms, float* best_ms) {
   if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
   if (!h->timing) return fail(HX_ERR_STATE, "created without opt.timing");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
-  HX_CUDA(cudaEventSynchronize(h->ev[3]));
+  if (back < 0 || back >= hx_sim::kTimedRuns || back >= h->runs)
+    return fail(HX_ERR_INVALID, "back must be 0 .. min(runs, " + std::to_string(hx_sim::kTimedRuns) + ") - 1");
+  cudaEvent_t* ev = h->run_ev(h->runs - 1 - back);
+  HX_CUDA(cudaEventSynchronize(ev[3]));
   float a = 0, b = 0, c = 0;
-  HX_CUDA(cudaEventElapsedTime(&a, h->ev[0], h->ev[1]));
-  HX_CUDA(cudaEventElapsedTime(&b, h->ev[1], h->ev[2]));
-  HX_CUDA(cudaEventElapsedTime(&c, h->ev[2], h->ev[3]));
+  HX_CUDA(cudaEventElapsedTime(&a, ev[0], ev[1]));
+  HX_CUDA(cudaEventElapsedTime(&b, ev[1], ev[2]));
+  HX_CUDA(cudaEventElapsedTime(&c, ev[2], ev[3]));
   if (prep_ms) *prep_ms = a;
   if (sim_ms) *sim_ms = b;
   if (best_ms) *best_ms = c;
@@ -914,22 +960,28 @@ namespace {
 
 __device__ __align__(256) unsigned char hx_static_scratch[HX_STATIC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
 std::mutex g_static_mu;
 unsigned char* g_static_base[kMaxDevices] = {};
 
-// Device address of hx_static_scratch on the current device, looked up once
-// per device (the host-side symbol is only a stand-in and must never be
-// passed to a kernel).
-int static_base(unsigned char** out) {
+// Device address of hx_static_scratch on the current device (the host-side
+// symbol is only a stand-in and must never be passed to a kernel).  It is
+// looked up again on every call made while `s` is not capturing, so a
+// device reset between calls cannot leave a stale address behind; a call
+// made during stream capture uses the address of the last earlier call on
+// this device, and fails if there was none.
+int static_base(cudaStream_t s, unsigned char** out) {
   int dev = 0;
   HX_CUDA(cudaGetDevice(&dev));
   if (dev < 0 || dev >= kMaxDevices) return fail(HX_ERR_INVALID, "device index out of range");
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  HX_CUDA(cudaStreamIsCapturing(s, &cap));
   std::lock_guard<std::mutex> lock(g_static_mu);
-  if (!g_static_base[dev]) {
+  if (cap == cudaStreamCaptureStatusNone) {
     void* p = nullptr;
     HX_CUDA(cudaGetSymbolAddress(&p, hx_static_scratch));
     g_static_base[dev] = static_cast<unsigned char*>(p);
+  } else if (!g_static_base[dev]) {
+    return fail(HX_ERR_STATE, "the first hx_sim_run_static call on a device must come before any stream capture");
   }
   *out = g_static_base[dev];
   return HX_OK;
@@ -1000,10 +1052,11 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   HX_CUDA(cudaGetDevice(&dev));
   HX_CUDA(cudaGetDeviceProperties(&prop, dev));
   const int smem_per_block = hx::kWarpsPerBlock * ck.smem_per_warp;
-  HX_CUDA(cudaFuncSetAttribute(hx::hx_sim_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_per_block));
+  const bool generic = needs_generic(grid, ck, false, false, false);
+  const void* kfn = generic ? (const void*)hx::hx_sim_kernel : (const void*)hx::hx_sim_kernel_lean;
+  if ((rc = ensure_dyn_smem(generic, smem_per_block))) return rc;
   int bps = 0;
-  HX_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, hx::hx_sim_kernel, hx::kWarpsPerBlock * 32,
-                                                        smem_per_block));
+  HX_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, kfn, hx::kWarpsPerBlock * 32, smem_per_block));
   if (bps < 1) return fail(HX_ERR_CUDA, "simulation kernel does not fit on an SM");
   int64_t blocks = std::min<int64_t>((int64_t)bps * prop.multiProcessorCount, fit_warps / hx::kWarpsPerBlock);
   blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (P + hx::kWarpsPerBlock - 1) / hx::kWarpsPerBlock));
@@ -1013,7 +1066,7 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   const int64_t o_topk = o_chains + warps * chains_per_warp;
 
   unsigned char* sb = nullptr;
-  if ((rc = static_base(&sb))) return rc;
+  if ((rc = static_base(s, &sb))) return rc;
   auto at = [&](int64_t off) { return static_cast<void*>(sb + off); };
   const int64_t offs[4] = {0, nq, 0, nc};
   HX_CUDA(cudaMemcpyAsync(at(o_qoff), offs, 2 * sizeof(int64_t), cudaMemcpyHostToDevice, s));
@@ -1104,7 +1157,10 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
 
   hx::hx_prep_kernel<<<(unsigned)std::max<int64_t>(1, (nq + 255) / 256), 256, 0, s>>>(pa, ck);
   HX_CUDA(cudaGetLastError());
-  hx::hx_sim_kernel<<<(unsigned)blocks, hx::kWarpsPerBlock * 32, smem_per_block, s>>>(sa, ck);
+  if (generic)
+    hx::hx_sim_kernel<<<(unsigned)blocks, hx::kWarpsPerBlock * 32, smem_per_block, s>>>(sa, ck);
+  else
+    hx::hx_sim_kernel_lean<<<(unsigned)blocks, hx::kWarpsPerBlock * 32, smem_per_block, s>>>(sa, ck);
   HX_CUDA(cudaGetLastError());
   hx::hx_best_kernel<<<2, 256, 0, s>>>(ba);
   HX_CUDA(cudaGetLastError());

@@ -114,6 +114,7 @@ def load(path: Optional[str] = None):
                        ("hx_sim_run", [vp, vp]), ("hx_sim_results", [vp, vp, sz]),
                        ("hx_sim_best", [vp, i32, vp]), ("hx_sim_records", [vp, i32, vp, vp, vp, vp, vp, sz]),
                        ("hx_sim_prep", [vp, i32, vp, vp, vp, vp, sz]), ("hx_sim_timings", [vp, vp, vp, vp]),
+                       ("hx_sim_timings_back", [vp, i32, vp, vp, vp]),
                        ("hx_sim_info", [vp, vp]), ("hx_sim_destroy", [vp]),
                        ("hx_sim_run_static", [vp, vp, vp, i32, vp, vp, vp]),
                        ("hx_selftest_div", [vp, vp, vp, vp, sz]),
@@ -322,9 +323,12 @@ class Sim:
                                               _p(out["tbar"]), _p(out["deadline"]), n))
         return out
 
-    def timings(self):
+    def timings(self, back: int = 0):
+        """(prep, simulate, best) milliseconds of the last run, or of the run
+        `back` runs before it (the handle keeps its last 64 runs)."""
         a, b, c = ctypes.c_float(), ctypes.c_float(), ctypes.c_float()
-        _check(self.lib, self.lib.hx_sim_timings(self.h, ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
+        _check(self.lib, self.lib.hx_sim_timings_back(self.h, int(back), ctypes.byref(a), ctypes.byref(b),
+                                                      ctypes.byref(c)))
         return float(a.value), float(b.value), float(c.value)
 
     def info(self) -> dict:

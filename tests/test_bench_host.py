@@ -37,3 +37,23 @@ def test_traffic_only_for_the_ceiling_workload():
     assert bench._is_ceiling(_args())
     for kw in (dict(recipe="3"), dict(traces=8), dict(queries=100), dict(alpha="1"), dict(policy="wb-pq")):
         assert not bench._is_ceiling(_args(**kw)), kw
+
+
+def test_stratified_sample_is_even_over_alpha():
+    wl = W.make_workload(3, n_traces=4, n_queries=10)
+    sims = bench.stratified_sims(wl, 256, 7)
+    assert len(sims) == len(set(sims)) == 256
+    a = wl.grid.alpha_fp[np.asarray(sims) % wl.grid.n_points]
+    vals, cnt = np.unique(a, return_counts=True)
+    assert vals.size == 8 and (cnt == 32).all()
+    assert len(set(np.asarray(sims) // wl.grid.n_points)) == 4
+    assert bench.stratified_sims(wl, wl.n_sims, 7) == list(range(wl.n_sims))
+
+
+def test_cpu_baseline_times_every_simulation_of_a_small_workload():
+    args = _args(recipe="0", queries=30)
+    wl = bench._workload(args)
+    cb = bench.cpu_baseline(args, wl, wl.n_sims)
+    assert cb["whole_workload"] and cb["sims"] == wl.n_sims and cb["kind"] == "oracle"
+    assert cb["value"] > 0 and cb["single_core"]["value"] > 0
+    assert abs(cb["events_per_s"] / cb["value"] - wl.traces[0].n_calls) < 1e-6 * wl.traces[0].n_calls

@@ -262,51 +262,74 @@ def test_upload_with_tenants():
 
 
 # ------------------------------------------------------------------ full size
-@pytest.mark.parametrize("cfg,n_sample", [(1, None), (2, 48), (3, 24)])
-def test_full_recipes_sampled(cfg, n_sample):
-    wl = W.make_workload(cfg)
+def stratified_sims(wl, per_alpha, alpha1_trace, seed):
+    """Simulations drawn evenly over the grid's alpha values (per_alpha of
+    each, trace and the other axes at random, without repeats), plus every
+    alpha = 1 point of one trace: the points whose local queues grow longest
+    and whose simulations cost the oracle the most."""
+    g = wl.grid
+    P, T = g.n_points, len(wl.traces)
+    rng = np.random.default_rng(seed)
+    sims = set()
+    for a in np.unique(g.alpha_fp):
+        pts = np.nonzero(g.alpha_fp == a)[0]
+        pick = rng.choice(T * pts.size, size=min(per_alpha, T * pts.size), replace=False)
+        sims.update((pick // pts.size * P + pts[pick % pts.size]).tolist())
+    a1 = np.nonzero(g.alpha_fp == W.SCALE)[0]
+    sims.update((alpha1_trace * P + a1).tolist())
+    return sorted(sims)
+
+
+def test_recipe1_full_every_sim():
+    wl = W.make_workload(1)
     sim = gpu(wl)
     g = sim.results()
-    nq = np.repeat([t.n_queries for t in wl.traces], wl.grid.n_points)
-    nc = np.repeat([t.n_calls for t in wl.traces], wl.grid.n_points)
-    assert (g["status"] == 0).all() and (g["n_done"] == nq).all() and (g["events"] == nc).all()
-    if n_sample is None:
-        sims = list(range(wl.n_sims))
-    else:
-        rng = np.random.default_rng(100 + cfg)
-        sims = sorted(set(rng.choice(wl.n_sims, n_sample, replace=False).tolist() + [wl.n_sims - 1]))
-    o = oracle_results(wl, sims)
-    assert_same(g[sims], o, f"recipe {cfg} sample")
-    nqt = [t.n_queries for t in wl.traces]
-    for obj in (W.OBJ_P95, W.OBJ_P95_SLO95):
-        gp, gs, per = oracle.best(g, len(wl.traces), wl.grid.n_points, nqt, obj)
-        bp, bs, _, bper = sim.best(obj)
-        assert (bp, bs) == (gp, gs) and bper.tolist() == per.tolist()
+    o = oracle_results(wl, range(wl.n_sims))
+    assert_same(g, o, "recipe 1")
+    check_best(sim, wl, o)
     sim.close()
 
 
-def test_full_size_ceiling_sampled():
-    """The benchmarked workload (256 traces x 20000 queries x 1024 points) in
-    the benchmark's launch configuration: every simulation completes, a
-    seeded sample matches the oracle exactly, and the best-point kernel agrees
-    with the oracle's rule applied to the GPU's result table."""
-    wl = W.make_workload(4)
+@pytest.mark.parametrize("cfg", [2, 3, 4])
+def test_full_size_stratified(cfg):
+    """A full recipe (config 4 is the benchmarked workload: 256 traces x
+    20000 queries x 1024 points) in the benchmark's launch configuration:
+    every simulation completes; a sample stratified over alpha (32 per alpha
+    value, over all traces) plus every alpha = 1 point of one full-length
+    trace matches the oracle exactly; the best-point kernel agrees with the
+    oracle's rule applied to the GPU's whole table; and five full-length
+    simulations (alpha = 0, two interior points, two at alpha = 1) have
+    per-call logs equal to the oracle's."""
+    wl = W.make_workload(cfg)
     sim = gpu(wl)
+    assert sim.info()["generic_kernel"] == 0
     g = sim.results()
     P = wl.grid.n_points
     nq = np.repeat([t.n_queries for t in wl.traces], P)
     nc = np.repeat([t.n_calls for t in wl.traces], P)
     assert (g["status"] == 0).all() and (g["n_done"] == nq).all() and (g["events"] == nc).all()
-    rng = np.random.default_rng(4)
-    sims = sorted(set(rng.choice(wl.n_sims, 12, replace=False).tolist() + [P - 1, wl.n_sims - 1, 37 * P + 1023]))
+    T = len(wl.traces)
+    sims = stratified_sims(wl, 32, T - 1, 100 + cfg)
+    assert len(sims) >= 256 and (wl.grid.alpha_fp[np.asarray(sims) % P] == W.SCALE).sum() >= P // 8
     o = oracle_results(wl, sims)
-    assert_same(g[sims], o, "recipe 4 sample")
+    assert_same(g[sims], o, f"recipe {cfg} stratified sample")
     nqt = [t.n_queries for t in wl.traces]
     for obj in (W.OBJ_P95, W.OBJ_P95_SLO95):
-        gp, gs, per = oracle.best(g, len(wl.traces), P, nqt, obj)
+        gp, gs, per = oracle.best(g, T, P, nqt, obj)
         bp, bs, _, bper = sim.best(obj)
         assert (bp, bs) == (gp, gs) and bper.tolist() == per.tolist()
     sim.close()
+    # full per-call logs of five full-length simulations (run alone as a subset)
+    a1 = np.nonzero(wl.grid.alpha_fp == W.SCALE)[0]
+    inner = np.nonzero((wl.grid.alpha_fp > 0) & (wl.grid.alpha_fp < W.SCALE))[0]
+    rng = np.random.default_rng(7 + cfg)
+    logged = sorted({0 * P + 0, 3 * P + int(rng.choice(inner)), (T // 2) * P + int(rng.choice(inner)),
+                     1 * P + int(a1[0]), (T - 2) * P + int(a1[-1])})
+    rec = gpu(wl, record=logged, subset=logged)
+    assert_same(rec.results()[logged], g[logged], f"recipe {cfg} logged runs vs the full run")
+    for j in range(len(logged)):
+        assert_logs(rec, wl, j)
+    rec.close()
 
 
 def test_point_sums_and_best_of_sums():
