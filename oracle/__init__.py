@@ -21,7 +21,8 @@ _LIB = os.path.join(_HERE, "libhxoracle.so")
 RESULT_DTYPE = np.dtype([("p95_us", "<i8"), ("makespan_us", "<i8"), ("events", "<i8"),
                          ("digest", "<u8"), ("slo_met", "<i4"), ("n_done", "<i4"),
                          ("status", "<i4"), ("pad", "<i4")])
-EXTRA_DTYPE = np.dtype([("slo_met", "<i4", (4,)), ("n_done", "<i4", (4,)), ("reissued", "<i4"), ("pad", "<i4")])
+EXTRA_DTYPE = np.dtype([("slo_met", "<i4", (4,)), ("n_done", "<i4", (4,)), ("reissued", "<i4"), ("pad", "<i4"),
+                        ("p95_us", "<i8", (4,))])
 FAULT_DTYPE = np.dtype([("inst", "<i4"), ("pad", "<i4"), ("t0_us", "<i8"), ("t1_us", "<i8"), ("slow_fp", "<i8")])
 
 

@@ -437,7 +437,10 @@ static int check_invariants(const sim_t* s) {
 int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt, int check,
                  hxo_result* res, const hxo_log* log, hxo_extra* ext) {
   memset(res, 0, sizeof(*res));
-  if (ext) memset(ext, 0, sizeof(*ext));
+  if (ext) {
+    memset(ext, 0, sizeof(*ext));
+    for (int t = 0; t < HXO_MAX_TENANTS; ++t) ext->p95_us[t] = -1;
+  }
   res->p95_us = -1;
   if (!validate(tr, cl) || pt->alpha_fp < 0 || pt->alpha_fp > FP_ONE || pt->beta_us2 < 0 ||
       pt->gamma_fp < 0 || pt->rho < 0 || pt->local_policy < 0 || pt->local_policy > 2 ||
@@ -467,6 +470,8 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
   s.waiting = (ivec*)calloc((size_t)N, sizeof(ivec));
   s.running = (ivec*)calloc((size_t)N, sizeof(ivec));
   int64_t* lat = (int64_t*)calloc(nq1, sizeof(int64_t));
+  uint8_t* lat_tenant = (uint8_t*)calloc(nq1, 1);  /* tenant of lat[j] */
+  int64_t* tlat = (int64_t*)calloc(nq1, sizeof(int64_t));
   int64_t* est_tmp = (int64_t*)calloc(nc1 * (size_t)cl->n_types, sizeof(int64_t));
   int64_t* svc_tmp = (int64_t*)calloc(nc1 * (size_t)cl->n_types, sizeof(int64_t));
   int64_t* tbar_tmp = (int64_t*)calloc(nc1, sizeof(int64_t));
@@ -475,7 +480,8 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
   int32_t bufcap = 0;
   int status = HXO_OK;
   if (!s.t_slo || !s.chains_left || !s.qid || !s.state || !s.inst || !s.enq || !s.budget || !s.remaining || !s.start ||
-      !s.end || !s.failed || !s.q || !s.waiting || !s.running || !lat || !est_tmp || !svc_tmp || !tbar_tmp) {
+      !s.end || !s.failed || !s.q || !s.waiting || !s.running || !lat || !lat_tenant || !tlat || !est_tmp ||
+      !svc_tmp || !tbar_tmp) {
     status = HXO_ERR_OOM;
     goto done;
   }
@@ -543,6 +549,7 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
       } else {
         int64_t l = now - tr->arrival_us[i];
         int ten = tr->tenant ? tr->tenant[i] : 0;
+        lat_tenant[n_done] = (uint8_t)ten;
         lat[n_done++] = l;
         t_done[ten]++;
         if (l <= s.t_slo[i]) {
@@ -575,6 +582,20 @@ int hxo_simulate(const hxo_trace* tr, const hxo_cluster* cl, const hxo_point* pt
       ext->n_done[t] = t_done[t];
     }
     ext->reissued = s.reissued;
+    /* per tenant, the nearest-rank P95 of its own queries' latencies */
+    for (int t = 0; t < HXO_MAX_TENANTS; ++t) {
+      int32_t n = 0;
+      for (int32_t j = 0; j < n_done; ++j)
+        if (lat_tenant[j] == t) tlat[n++] = lat[j];
+      if (status != HXO_OK) {
+        ext->p95_us[t] = -1;
+      } else if (n == 0) {
+        ext->p95_us[t] = 0;
+      } else {
+        qsort(tlat, (size_t)n, sizeof(int64_t), cmp_i64);
+        ext->p95_us[t] = tlat[(95 * (int64_t)n + 99) / 100 - 1];
+      }
+    }
   }
   res->makespan_us = makespan;
   res->events = events;
@@ -605,7 +626,7 @@ done:
     for (int m = 0; m < N; ++m) free(s.running[m].v);
   free(s.t_slo); free(s.chains_left); free(s.qid); free(s.state); free(s.inst); free(s.enq);
   free(s.budget); free(s.remaining); free(s.start); free(s.end); free(s.failed); free(s.q); free(s.waiting); free(s.running);
-  free(lat); free(est_tmp); free(svc_tmp); free(tbar_tmp); free(ubuf); free(ebuf); free(rbuf);
+  free(lat); free(lat_tenant); free(tlat); free(est_tmp); free(svc_tmp); free(tbar_tmp); free(ubuf); free(ebuf); free(rbuf);
   return status;
 }
 

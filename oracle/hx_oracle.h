@@ -91,6 +91,8 @@ typedef struct {
   int32_t n_done[HXO_MAX_TENANTS];
   int32_t reissued;
   int32_t pad;
+  int64_t p95_us[HXO_MAX_TENANTS]; /* nearest-rank P95 of each tenant's query latencies
+                                      (0 for a tenant without queries, -1 if failed) */
 } hxo_extra;
 
 /* Per-call estimates of Eq. (comp) and the mean over instances, and the

@@ -45,6 +45,12 @@ def _mix64(z):
     return z ^ (z >> 31)
 
 
+def _p95(lat):
+    """Nearest-rank P95 of a latency list sorted here (0 for none)."""
+    s = np.sort(np.asarray(lat, np.int64))
+    return int(s[-(-95 * s.size // 100) - 1]) if s.size else 0
+
+
 def _slowdown(cl, inst, start):
     """slow_fp of the first fault window covering each (instance, start), else 0."""
     slow = np.zeros(inst.shape[0], np.int64)
@@ -210,6 +216,7 @@ def test_tenants_and_single_shots(name):
             sel = tr.tenant == t
             assert int(ext["n_done"][t]) == int(sel.sum())
             assert int(ext["slo_met"][t]) == int(np.sum(lat[sel] <= p["t_slo"][sel]))
+            assert int(ext["p95_us"][t]) == _p95(lat[sel])
         assert int(ext["slo_met"].sum()) == int(res["slo_met"])
     if name.startswith("competing"):
         single = tr.k == 0
@@ -296,3 +303,4 @@ def test_invariants_random_workloads(seed, lean):
             sel = ten == t
             assert int(ext["n_done"][t]) == int(sel.sum())
             assert int(ext["slo_met"][t]) == int(np.sum(lat[sel] <= p["t_slo"][sel]))
+            assert int(ext["p95_us"][t]) == _p95(lat[sel])

@@ -31,6 +31,8 @@ def test_hand_case(name):
         assert ext["slo_met"].tolist() == exp["tenant_slo_met"]
         assert ext["n_done"].tolist() == exp["tenant_done"]
         assert int(ext["reissued"]) == exp["reissued"]
+    if "tenant_p95_us" in exp:
+        assert ext["p95_us"].tolist() == exp["tenant_p95_us"]
 
 
 def test_table2_pick():
@@ -97,6 +99,37 @@ def test_closed_form_fcfs_burst(n):
     assert int(res["p95_us"]) == (2 * n + rank) * s
     # T_slo = 3 * (3 s): met iff 2n + j + 1 <= 9
     assert int(res["slo_met"]) == sum(1 for j in range(n) if 2 * n + j + 1 <= 9)
+
+
+@pytest.mark.parametrize("n,n_tenants", [(1, 2), (5, 2), (40, 2), (41, 3), (200, 4)])
+def test_closed_form_fcfs_burst_per_tenant(n, n_tenants):
+    """The burst above with query j in tenant j mod n_tenants: tenant t holds
+    queries j = t, t + n_tenants, ... in latency order, so its P95 is the
+    latency (2n + j + 1) s of its ceil(0.95 n_t)-th query, and a tenant
+    without queries reports 0; SLO counts split the same way."""
+    s = 1000
+    tr, cl1 = cases.uniform_single_instance(n, [0] * n, svc_us=s)
+    tr.tenant = (np.arange(n) % n_tenants).astype(np.uint8)
+    mult = np.full(n_tenants, 3 * W.SCALE, np.int64)
+    cl = W.Cluster(cl1.prefill_tok_s, cl1.decode_us_tok, cl1.slots, cl1.inst_type, cl1.ref_type, cl1.slo_mult_fp,
+                   cl1.rmax, cl1.stage_ref_prompt, cl1.stage_ref_out, mult)
+    pt = dict(alpha_fp=W.SCALE // 2, gamma_fp=W.SCALE, beta_us2=10 ** 6, rho=0, local_policy=1,
+              dispatch_policy=0)
+    res, ext = oracle.simulate(tr, cl, pt, check=True, extra=True)
+    assert res["status"] == 0
+    for t in range(4):
+        js = [j for j in range(n) if j % n_tenants == t] if t < n_tenants else []
+        if not js:
+            assert int(ext["p95_us"][t]) == 0 and int(ext["n_done"][t]) == 0
+            continue
+        j = js[-(-95 * len(js) // 100) - 1]
+        assert int(ext["p95_us"][t]) == (2 * n + j + 1) * s
+        assert int(ext["n_done"][t]) == len(js)
+        assert int(ext["slo_met"][t]) == sum(1 for q in js if 2 * n + q + 1 <= 9)
+    # with one tenant the tenant's P95 is the simulation's
+    tr.tenant = None
+    res1, ext1 = oracle.simulate(tr, cl1, pt, extra=True)
+    assert int(ext1["p95_us"][0]) == int(res1["p95_us"]) and ext1["p95_us"][1:].tolist() == [0, 0, 0]
 
 
 @pytest.mark.parametrize("policy", [0, 1])
