@@ -203,13 +203,17 @@ typedef struct hx_best {
   int32_t* per_trace_point;   /* caller-owned [n_traces], may be NULL */
 } hx_best;
 
-/* Per-simulation counts beside hx_result: SLO hits and completed queries
- * per tenant, and the attempts that timed out and were re-issued. */
+/* Per-simulation counts beside hx_result (Sec. 5's multi-tenant
+ * evaluation): SLO hits, completed queries and the nearest-rank P95 of query
+ * latency per tenant, and the attempts that timed out and were re-issued. */
 typedef struct hx_extra {
   int32_t slo_met[HX_MAX_TENANTS];
   int32_t n_done[HX_MAX_TENANTS];
   int32_t reissued;
   int32_t pad;
+  int64_t p95_us[HX_MAX_TENANTS];  /* sorted L_t[ceil(0.95 n_t) - 1] over tenant t's queries;
+                                      0 for a tenant without queries, -1 if the simulation
+                                      failed or was skipped */
 } hx_extra;
 
 typedef struct hx_sim hx_sim;

@@ -123,6 +123,9 @@ struct hx_sim {
   hx::BestCand* d_best_trace = nullptr;
   hx::BestCand* d_best_global = nullptr;
   int64_t* d_point_sums = nullptr;
+  // per-tenant top-K heaps (generic kernel with several tenants)
+  int32_t* d_tenant_kcap = nullptr;
+  int64_t tenant_topk_off[HX_MAX_TENANTS] = {0, 0, 0, 0};
   // device: scratch
   hx::HeapEnt* d_arena = nullptr;
   uint8_t* d_chains = nullptr;
@@ -314,6 +317,19 @@ int upload(T* dst, const T* src, int64_t count, cudaStream_t s) {
   return HX_OK;
 }
 
+// Top-K size of each (trace, tenant) for the per-tenant P95: n_t - ceil(0.95 n_t) + 1
+// over the tenant's n_t queries (0 without queries); at most the trace's own K.
+std::vector<int32_t> tenant_kcaps(const hx_trace* traces, int32_t n_traces) {
+  std::vector<int32_t> k((size_t)n_traces * HX_MAX_TENANTS, 0);
+  for (int t = 0; t < n_traces; ++t) {
+    int32_t n[HX_MAX_TENANTS] = {0, 0, 0, 0};
+    for (int32_t i = 0; i < traces[t].n_queries; ++i) n[traces[t].tenant ? traces[t].tenant[i] : 0]++;
+    for (int u = 0; u < HX_MAX_TENANTS; ++u)
+      k[(size_t)t * HX_MAX_TENANTS + u] = n[u] ? n[u] - (95 * n[u] + 99) / 100 + 1 : 0;
+  }
+  return k;
+}
+
 // Copies the per-call and per-query trace arrays of all traces to the device.
 int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
   std::vector<int64_t> arrival((size_t)h->n_q), qcall((size_t)h->n_q + 1);
@@ -344,6 +360,11 @@ int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
         (rc = upload(h->d_retry + co, tr.retry, tr.n_calls, s)))
       return rc;
     co += tr.n_calls;
+  }
+  std::vector<int32_t> kcap;
+  if (h->d_tenant_kcap) {
+    kcap = tenant_kcaps(traces, h->n_traces);
+    if ((rc = upload(h->d_tenant_kcap, kcap.data(), (int64_t)kcap.size(), s))) return rc;
   }
   // the host staging vectors die here: the copies must finish first
   HX_CUDA(cudaStreamSynchronize(s));
@@ -390,9 +411,10 @@ void fill_cluster(const hx_cluster* cluster, hx::ClusterK& ck) {
   }
   ck.total_slots = base;
   // per-tenant SLO multipliers replace slo_mult_fp when given
-  ck.n_tenants = cluster->tenant_slo_mult_fp ? std::max(cluster->n_tenants, 1) : 0;
+  ck.n_tenants = std::max(cluster->n_tenants, 1);
   for (int t = 0; t < HX_MAX_TENANTS; ++t)
-    ck.tenant_mult[t] = t < ck.n_tenants ? cluster->tenant_slo_mult_fp[t] : cluster->slo_mult_fp;
+    ck.tenant_mult[t] = (cluster->tenant_slo_mult_fp && t < ck.n_tenants) ? cluster->tenant_slo_mult_fp[t]
+                                                                          : cluster->slo_mult_fp;
   ck.timeout_mult_fp = cluster->timeout_mult_fp;
   ck.n_faults = cluster->n_faults;
   for (int f = 0; f < cluster->n_faults; ++f) {
@@ -557,6 +579,17 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   if (opt && opt->arena_entries > 0) h->arena_per_warp = opt->arena_entries;
   h->chains_per_warp = align_up(std::max(h->max_nq, 1), 256);
   h->topk_per_warp = align_up(h->max_kcap, 32);
+  if (h->generic && ck.n_tenants > 1) {
+    // one more heap per tenant after the simulation's own, each sized for a
+    // whole trace (a tenant's K never exceeds its trace's), so uploads of new
+    // tenant assignments need no reallocation
+    for (int t = 0; t < HX_MAX_TENANTS; ++t) h->tenant_topk_off[t] = h->topk_per_warp * (1 + t);
+    h->topk_per_warp *= 1 + HX_MAX_TENANTS;
+    if ((rc = h->alloc(&h->d_tenant_kcap, (int64_t)n_traces * HX_MAX_TENANTS))) return bail(rc);
+    const std::vector<int32_t> kcap = tenant_kcaps(traces, n_traces);
+    if ((rc = upload(h->d_tenant_kcap, kcap.data(), (int64_t)kcap.size(), s0))) return bail(rc);
+    if (cudaStreamSynchronize(s0) != cudaSuccess) return bail(fail(HX_ERR_CUDA, "tenant upload failed"));
+  }
   const int64_t w = h->resident_warps;
   if ((rc = h->alloc(&h->d_arena, w * h->arena_per_warp)) || (rc = h->alloc(&h->d_chains, w * h->chains_per_warp)) ||
       (rc = h->alloc(&h->d_topk, w * h->topk_per_warp)))
@@ -677,6 +710,8 @@ int hx_sim_run(hx_sim* h, void* stream) {
   sa.rec_end = h->d_rec_end;
   sa.rec_stride = h->rec_stride;
   sa.extras = h->d_extras;
+  sa.tenant_kcap = h->d_tenant_kcap;
+  for (int t = 0; t < HX_MAX_TENANTS; ++t) sa.tenant_topk_off[t] = h->tenant_topk_off[t];
   sa.subset = h->d_subset;
   sa.n_work = h->n_work;
   sa.checked = h->checked ? 1 : 0;
@@ -739,6 +774,7 @@ int hx_sim_extras(hx_sim* h, hx_extra* host_out, size_t n) {
     hx_extra e{};
     e.slo_met[0] = res[i].slo_met;
     e.n_done[0] = res[i].n_done;
+    for (int t = 0; t < HX_MAX_TENANTS; ++t) e.p95_us[t] = res[i].status != HX_OK ? -1 : t == 0 ? res[i].p95_us : 0;
     host_out[i] = e;
   }
   return HX_OK;
@@ -1142,6 +1178,8 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   sa.rec_end = nullptr;
   sa.rec_stride = 0;
   sa.extras = nullptr;
+  sa.tenant_kcap = nullptr;
+  for (int t = 0; t < HX_MAX_TENANTS; ++t) sa.tenant_topk_off[t] = 0;
   sa.subset = nullptr;
   sa.n_work = P;
   sa.checked = 0;

@@ -129,6 +129,9 @@ struct SimArgs {
   int64_t* rec_end;
   int64_t rec_stride;
   hx_extra* extras;         // [n_sims] per-tenant counts and re-issues (generic kernel), or NULL
+  const int32_t* tenant_kcap;  // [n_traces * 4] top-K size per (trace, tenant) (0: no queries), or
+                               // NULL: one tenant
+  int64_t tenant_topk_off[HX_MAX_TENANTS];  // tenant t's top-K heap within the warp's topk slice
   const int64_t* subset;    // [n_work] sims to run in work order, or NULL: all n_sims
   int64_t n_work;
   int32_t checked;          // check the scheduler's invariants after every event (generic kernel)
@@ -163,7 +166,7 @@ struct WarpShared {
   int32_t nq, nc;
   int64_t sim, clk0;            // result index and start clock of the simulation
   uint64_t akey;                // next arrival's event key (written alike by every lane)
-  int32_t qa, pad0;             // arrivals taken so far (likewise)
+  int32_t qa, trace;            // arrivals taken so far (likewise); the simulation's trace
   // lane-0 accumulators
   uint64_t digest;
   int64_t makespan;
@@ -171,6 +174,8 @@ struct WarpShared {
   int64_t tkmin;                // root of the full top-K heap (written alike by every lane)
   longlong2 dterm[16];          // digest terms waiting to be hashed: (time, id tag)
   int32_t tslo[HX_MAX_TENANTS], tdone[HX_MAX_TENANTS];  // per-tenant counts (generic kernel)
+  int32_t ttk[HX_MAX_TENANTS];  // per-tenant top-K heaps: entries (generic kernel with tenants)
+  int64_t ttkmin[HX_MAX_TENANTS];  //                 and roots once full
   int32_t reissued, excl;       // timed-out attempts; the instance a re-issue avoids (-1: none)
   uint64_t slot[1];             // [total_slots], then with faults one fail flag byte per slot
 };

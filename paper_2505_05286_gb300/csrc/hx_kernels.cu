@@ -134,6 +134,7 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
       for (int t = 0; t < HX_MAX_TENANTS; ++t) {
         x.slo_met[t] = 0;
         x.n_done[t] = 0;
+        x.p95_us[t] = -1;
       }
       x.reissued = 0;
       x.pad = 0;
@@ -335,11 +336,12 @@ __device__ __noinline__ HeapEnt heap_sift_warp(HeapEnt* h, int m, HeapEnt sink, 
 // Min-heap of the K largest latencies seen so far, 32-ary like the local
 // queues; its root is the K-th largest latency, i.e. the nearest-rank P95
 // when K = n - ceil(0.95 n) + 1.  All lanes call with the same v: lane 0
-// writes the heap, every lane writes the same size and root copies.
-__device__ __noinline__ void topk_insert_warp(WarpShared* W, int64_t v, int lane) {
-  int64_t* const h = W->topk;
-  const int n = W->tk;
-  if (n < W->kcap) {
+// writes the heap, every lane writes the same size (*size) and root (*root)
+// copies in shared memory.
+__device__ __noinline__ void topk_insert_warp(int64_t* h, int32_t* size, int kcap, int64_t* root_out, int64_t v,
+                                              int lane) {
+  const int n = *size;
+  if (n < kcap) {
     // filling: sift up on lane 0 (few levels)
     if (lane == 0) {
       int i = n;
@@ -353,9 +355,9 @@ __device__ __noinline__ void topk_insert_warp(WarpShared* W, int64_t v, int lane
       h[i] = v;
     }
     __syncwarp();
-    W->tk = n + 1;
-    if (n + 1 == W->kcap) W->tkmin = h[0];
-  } else if (v > W->tkmin) {
+    *size = n + 1;
+    if (n + 1 == kcap) *root_out = h[0];
+  } else if (v > *root_out) {
     // v replaces the root and sinks; one lane per child (latencies are >= 0)
     int i = 0;
     int64_t root = v;
@@ -373,7 +375,7 @@ __device__ __noinline__ void topk_insert_warp(WarpShared* W, int64_t v, int lane
     }
     if (lane == 0) h[i] = v;
     __syncwarp();
-    W->tkmin = root;
+    *root_out = root;
   }
 }
 
@@ -476,7 +478,7 @@ __device__ __forceinline__ void finish_query(WarpShared* W, int& dn, int32_t qid
   digest_push(W, dn, now, query_tag(qid), lane);
   // most latencies of a full heap fall below its root and change nothing
   const int64_t v = now - arrival;
-  if (W->tk < W->kcap || v > W->tkmin) topk_insert_warp(W, v, lane);
+  if (W->tk < W->kcap || v > W->tkmin) topk_insert_warp(W->topk, &W->tk, W->kcap, &W->tkmin, v, lane);
 }
 
 __device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, int m, int64_t now, int64_t budget) {
@@ -542,6 +544,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       W->nq = nq;
       W->nc = nc;
       W->sim = sim;
+      W->trace = t;
       W->clk0 = clk0;
     }
 
@@ -600,6 +603,8 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       for (int t = 0; t < HX_MAX_TENANTS; ++t) {
         W->tslo[t] = 0;
         W->tdone[t] = 0;
+        W->ttk[t] = 0;
+        W->ttkmin[t] = 0;
       }
       W->reissued = 0;
       W->excl = -1;
@@ -745,12 +750,23 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           rel_count = k;
         } else if (stg == HX_STAGE_E) {
           const int64_t dl = r->deadline;
-          if (kGeneric && lane == 0) {
+          const int64_t arr = r->arrival;
+          if (kGeneric) {
             const int ten = (tail.w >> 8) & 0xff;
-            W->tdone[ten]++;
-            W->tslo[ten] += now <= dl ? 1 : 0;
+            if (lane == 0) {
+              W->tdone[ten]++;
+              W->tslo[ten] += now <= dl ? 1 : 0;
+            }
+            if (a.tenant_kcap) {
+              // this tenant's own top-K, for its P95 (Sec. 5's per-tenant tail latency)
+              const int kc = a.tenant_kcap[(int64_t)W->trace * HX_MAX_TENANTS + ten];
+              const int64_t v = now - arr;
+              __syncwarp();
+              if (W->ttk[ten] < kc || v > W->ttkmin[ten])
+                topk_insert_warp(W->topk + a.tenant_topk_off[ten], &W->ttk[ten], kc, &W->ttkmin[ten], v, lane);
+            }
           }
-          finish_query(W, dn, qid, now, r->arrival, dl, lane);
+          finish_query(W, dn, qid, now, arr, dl, lane);
         } else {
           const int32_t nx = tail.y;
           if (nx >= 0) {
@@ -956,6 +972,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         for (int t = 0; t < HX_MAX_TENANTS; ++t) {
           ex.slo_met[t] = W->tslo[t];
           ex.n_done[t] = W->tdone[t];
+          if (st != HX_OK) ex.p95_us[t] = -1;
+          else if (!a.tenant_kcap) ex.p95_us[t] = t == 0 ? res.p95_us : 0;
+          else ex.p95_us[t] = W->ttk[t] > 0 ? W->topk[a.tenant_topk_off[t]] : 0;
         }
         ex.reissued = W->reissued;
         ex.pad = 0;

@@ -29,7 +29,8 @@ OBJ_P95, OBJ_P95_SLO95 = 0, 1
 RESULT_DTYPE = np.dtype([("p95_us", "<i8"), ("makespan_us", "<i8"), ("events", "<i8"),
                          ("digest", "<u8"), ("slo_met", "<i4"), ("n_done", "<i4"),
                          ("status", "<i4"), ("cycles_k", "<i4")])
-EXTRA_DTYPE = np.dtype([("slo_met", "<i4", (4,)), ("n_done", "<i4", (4,)), ("reissued", "<i4"), ("pad", "<i4")])
+EXTRA_DTYPE = np.dtype([("slo_met", "<i4", (4,)), ("n_done", "<i4", (4,)), ("reissued", "<i4"), ("pad", "<i4"),
+                        ("p95_us", "<i8", (4,))])
 
 
 class HxError(RuntimeError):

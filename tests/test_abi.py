@@ -40,7 +40,7 @@ int main(void) {
   F(hx_cluster, stage_ref_out) F(hx_cluster, n_faults) F(hx_cluster, tenant_slo_mult_fp)
   F(hx_cluster, timeout_mult_fp) F(hx_cluster, faults)
   S(hx_fault) F(hx_fault, t0_us) F(hx_fault, slow_fp)
-  S(hx_extra) F(hx_extra, n_done) F(hx_extra, reissued)
+  S(hx_extra) F(hx_extra, n_done) F(hx_extra, reissued) F(hx_extra, p95_us)
   S(hx_grid) F(hx_grid, alpha_fp) F(hx_grid, dispatch_policy)
   S(hx_options) F(hx_options, record_sims) F(hx_options, timing) F(hx_options, force_generic)
   F(hx_options, n_subset) F(hx_options, sim_subset) F(hx_options, checked) F(hx_options, arena_entries)

@@ -380,7 +380,7 @@ def test_lean_and_generic_kernels_agree():
 
 
 def assert_extras(g, o, what=""):
-    for f in ("slo_met", "n_done", "reissued"):
+    for f in ("slo_met", "n_done", "reissued", "p95_us"):
         bad = np.nonzero((g[f] != o[f]).reshape(len(g), -1).any(axis=1))[0]
         assert bad.size == 0, f"{what} extra field {f} differs at {bad[:8].tolist()}"
 
@@ -500,12 +500,14 @@ def test_four_tenants_and_only_single_shots():
 
 def test_per_tenant_p95_from_records():
     """Per-tenant P95 from a recorded simulation's call end times equals the
-    oracle's, also when fault windows stretch services."""
+    oracle's and the device's own per-tenant P95, also when fault windows
+    stretch services."""
     from paper_2505_05286_gb300 import tenants as T
     for name, nq in (("two-tenant", 400), ("faulty", 1400)):
         wl = W.make_workload(name, n_traces=1, n_queries=nq)
         tr = wl.traces[0]
         sim = gpu(wl, record=[5, 40])
+        ex = sim.extras()
         for j, s in enumerate([5, 40]):
             _, lo = oracle.simulate(tr, wl.cluster, oracle.point_of(wl.grid, s), log=True)
             lat_g = T.query_latencies(tr, sim.records(j))
@@ -513,6 +515,21 @@ def test_per_tenant_p95_from_records():
             assert (lat_g == lat_o).all()
             nt = wl.cluster.n_tenants
             assert T.tenant_p95(lat_g, tr.tenant, nt) == T.tenant_p95(lat_o, tr.tenant, nt)
+            assert [int(x) for x in ex["p95_us"][s][:nt]] == [x or 0 for x in T.tenant_p95(lat_o, tr.tenant, nt)]
+        sim.close()
+
+
+def test_per_tenant_p95_on_the_grid_without_records():
+    """The device's per-tenant P95 on every simulation of the two-tenant and
+    competing recipes (no per-call logs), against the oracle's."""
+    for name, nt, nq in (("two-tenant", 2, 500), ("competing-50", 1, 400)):
+        wl = W.make_workload(name, n_traces=nt, n_queries=nq)
+        sim = gpu(wl)
+        o, oe = oracle.run(wl, range(wl.n_sims), procs=NPROC, extra=True)
+        assert_same(sim.results(), o, name)
+        ex = sim.extras()
+        assert_extras(ex, oe, name)
+        assert (ex["p95_us"][:, :2] > 0).all() and (ex["p95_us"][:, 2:] == 0).all()
         sim.close()
 
 
