@@ -77,7 +77,10 @@ enum {
   HX_ERR_STATE = 6,      /* call out of order (e.g. results before run) */
   HX_ERR_INVARIANT = 7,  /* a simulation broke a scheduler invariant (per-sim status;
                             a library bug, never expected) */
-  HX_SKIPPED = 8         /* not in the run's subset (per-sim status) */
+  HX_SKIPPED = 8,        /* not in the run's subset (per-sim status) */
+  HX_ERR_BOUNDS = 9      /* bounds-checked build only: an index the simulation formed was out
+                            of range; the access was skipped (per-sim status; a library bug,
+                            never expected) */
 };
 
 enum { HX_STAGE_S = 0, HX_STAGE_G = 1, HX_STAGE_C = 2, HX_STAGE_E = 3 };

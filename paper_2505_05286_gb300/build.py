@@ -14,24 +14,34 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libhxsim.so")
+# the bounds-checked build (-DHX_CHECKED): every index the simulation kernel
+# forms is range-checked, a failure is a per-simulation status (HX_ERR_BOUNDS)
+LIB_CHECKED = os.path.join(PKG, "libhxsim_checked.so")
 SOURCES = ["hx_kernels.cu", "hx_api.cu"]
 NVCC = os.environ.get("NVCC", "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 
 
-def _stale() -> bool:
-    if not os.path.exists(LIB):
+def _stale(out: str) -> bool:
+    if not os.path.exists(out):
         return True
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(out)
     deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC)] + [os.path.join(INCLUDE, "hxsim.h")]
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(force: bool = False, verbose: bool = False, extra=(), out: str = LIB) -> str:
-    if not force and out == LIB and not _stale():
-        return LIB
-    objdir = os.path.join(os.path.dirname(out), "_build" + ("" if out == LIB else "_" + os.path.basename(out)))
+def build(force: bool = False, verbose: bool = False, extra=(), out: str = LIB, checked: bool = True) -> str:
+    """Build `out` (default: libhxsim.so) and, with `checked`, the
+    bounds-checked libhxsim_checked.so beside it, in parallel."""
+    if out == LIB and checked:
+        with ThreadPoolExecutor(2) as ex:
+            jobs = [ex.submit(build, force, verbose, extra, LIB, False),
+                    ex.submit(build, force, verbose, tuple(extra) + ("-DHX_CHECKED",), LIB_CHECKED, False)]
+            return [j.result() for j in jobs][0]
+    if not force and out in (LIB, LIB_CHECKED) and not _stale(out):
+        return out
+    objdir = os.path.join(os.path.dirname(out), "_build" + ("" if out == LIB else "_" + os.path.splitext(os.path.basename(out))[0]))
     os.makedirs(objdir, exist_ok=True)
 
     def compile_one(src):

@@ -153,7 +153,8 @@ struct WarpShared {
   int32_t pest[HX_MAX_K];
   // per-simulation constants
   int32_t A, one_minus_a;        // alpha and 1 - alpha, fixed point
-  int32_t rewards, pad2;          // 1 when dispatch scores need the reward term
+  int32_t rewards, oob;          // 1 when dispatch scores need the reward term; an index check
+                                // failed (bounds-checked build)
   int64_t G, beta;
   float betaf, pad3;            // beta as a float (the reward quotient's numerator)
   int64_t frest[kFRows];        // rest-of-path cost of the budget denominator by fcode

@@ -494,6 +494,27 @@ __device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, i
 #ifndef HX_SIM_MIN_BLOCKS
 #define HX_SIM_MIN_BLOCKS 7
 #endif
+
+// Bounds-checked build (-DHX_CHECKED): before every shared- or global-memory
+// access whose index the simulation forms from its own state (instance,
+// request id, query id, slot count, heap offset and size, top-K size), the
+// index is range-checked; a failed check sets the simulation's status to
+// HX_ERR_BOUNDS and leaves the loop it is in instead of making the access,
+// and the simulation stops after that event.  Every checked value is the
+// same on all lanes, so the exit is warp-uniform.  In the normal build the
+// checks compile to nothing.
+#ifdef HX_CHECKED
+#define HX_BOUND(cond)          \
+  if (!(cond)) {                \
+    status = HX_ERR_BOUNDS;     \
+    break;                      \
+  }
+#define HX_STOP_IF_FAILED() \
+  if (status != HX_OK) break;
+#else
+#define HX_BOUND(cond)
+#define HX_STOP_IF_FAILED()
+#endif
 // Resident blocks per SM the register allocation aims for (4 warps each).
 template <bool kGeneric>
 __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
@@ -634,6 +655,12 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     // event bound; re-issued attempts add events while fault windows last
     const bool faults = kGeneric && c.n_faults > 0;
     int32_t steps_left = nc + nq + 8 + (faults ? 16 * nc + 4096 : 0);
+#ifdef HX_CHECKED
+    // the warp's scratch slices must hold this trace's chain counters and top-K
+    if (!(nq <= a.chains_per_warp && W->kcap <= a.topk_per_warp && (a.tenant_kcap == nullptr ||
+          (int64_t)(HX_MAX_TENANTS + 1) * a.tenant_topk_off[0] <= a.topk_per_warp)))
+      status = HX_ERR_BOUNDS;
+#endif
 
     // Request rid starts on instance m now and runs until now + svc: its key
     // joins the cn sorted keys of m's running calls at sl.
@@ -692,6 +719,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     };
 
     for (;;) {
+      HX_STOP_IF_FAILED()
       const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
       const uint64_t akey = W->akey;
       if (ck >= kNoEvent && akey == kKeyInf) break;
@@ -707,10 +735,13 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         // completion on instance m
         const int m = (int)(ck & 127ull);
         now = (int64_t)(ck >> 7);
+        HX_BOUND(m < N)
         uint64_t* const sl = W->slot + c.slot_base[m];
         const int cn = W->cnt[m];
+        HX_BOUND(cn >= 1 && cn <= c.inst_slots[m] && c.slot_base[m] + cn <= c.total_slots)
         // the finishing call heads m's sorted slots
         const int32_t rid = (int32_t)(sl[0] & 0xffffffull);
+        HX_BOUND(rid < nc)
         // the finished call's record: issued now, used after the slot shift
         const CallRec* r = rec + rid;
         const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
@@ -737,6 +768,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         if (hs_m > 0) touched |= 1ull << m;
         const int stg = tail.w & 0xff;
         const int32_t qid = tail.z;
+        HX_BOUND(qid >= 0 && qid < nq)
         if (faults && failed) {
           // the attempt timed out: the request goes out again, avoiding m
           if (lane == 0) W->reissued++;
@@ -745,6 +777,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           rel_count = 1;
         } else if (stg == HX_STAGE_S) {
           const int k = (tail.w >> 16) & 0xff;
+          HX_BOUND(k >= 1 && k <= HX_MAX_K && rid + k < nc)
           if (lane == 0) W->chains[qid] = (uint8_t)k;
           rel_first = rid + 1;
           rel_count = k;
@@ -753,6 +786,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           const int64_t arr = r->arrival;
           if (kGeneric) {
             const int ten = (tail.w >> 8) & 0xff;
+            HX_BOUND(ten < HX_MAX_TENANTS)
             if (lane == 0) {
               W->tdone[ten]++;
               W->tslo[ten] += now <= dl ? 1 : 0;
@@ -760,6 +794,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             if (a.tenant_kcap) {
               // this tenant's own top-K, for its P95 (Sec. 5's per-tenant tail latency)
               const int kc = a.tenant_kcap[(int64_t)W->trace * HX_MAX_TENANTS + ten];
+              HX_BOUND(W->trace < a.n_traces && kc <= a.tenant_topk_off[0])
               const int64_t v = now - arr;
               __syncwarp();
               if (W->ttk[ten] < kc || v > W->ttkmin[ten])
@@ -769,6 +804,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           finish_query(W, dn, qid, now, arr, dl, lane);
         } else {
           const int32_t nx = tail.y;
+          HX_BOUND(nx >= 0 ? nx < nc : ~nx < nc)
           if (nx >= 0) {
             rel_first = nx;
             rel_count = 1;
@@ -785,7 +821,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         now = (int64_t)(akey >> 7);
         const int64_t qbase = W->qb;
         const int32_t qa = W->qa;
+        HX_BOUND(qa < W->nq)
         rel_first = (int32_t)(a.qcall[qbase + qa] - W->cb);
+        HX_BOUND(rel_first >= 0 && rel_first < nc)
         rel_count = 1;
         W->qa = qa + 1;
         W->akey = qa + 1 < W->nq ? (((uint64_t)a.arrival[qbase + qa + 1] << 7) | kArrivalTag) : kKeyInf;
@@ -796,6 +834,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       // batch boundary below, and only if it has to wait).
       for (int32_t jr = 0; jr < rel_count; ++jr) {
         const int32_t rid = rel_first + jr;
+        HX_BOUND(rid < nc)
         const CallRec* r = rec + rid;
         // Eq. (comp) and the service time on this lane's two instances
         const int e0 = r->est[ty0], e1 = r->est[ty1];
@@ -832,6 +871,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           m = warp_argmax_s64(take1 ? s1 : s0, take1 ? m1 : m0);
         }
         if (kGeneric) W->excl = -1;
+        HX_BOUND(m >= 0 && m < N)
         // the winner's costs, from the lane that owns it
         const int64_t est_m = __shfl_sync(kFull, m < 32 ? e0 : e1, m & 31);
         const int svc_m = __shfl_sync(kFull, m < 32 ? v0 : v1, m & 31);
@@ -844,6 +884,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         if (kGeneric) {
           const int recj = W->recj;
           if (recj >= 0) {
+            HX_BOUND(rid < a.rec_stride)
             const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
             const int64_t budget = slo_budget(r->deadline - now, tail.x, tail.x + W->frest[(uint32_t)tail.w >> 24]);
             if (lane == 0) log_dispatch(a, recj, rid, m, now, budget);
@@ -865,6 +906,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           }
         }
         // the local-queue key is formed only if the request has to wait
+        HX_BOUND(npend < HX_MAX_K)
         if (lane == npend) {
           pend_m = m;
         }
@@ -875,6 +917,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         npend++;
         touched |= 1ull << m;
       }
+      HX_STOP_IF_FAILED()
 
       // Batch boundary on every touched instance: its free slots go to the most
       // urgent of the waiting requests and this event's new ones.
@@ -882,6 +925,15 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       while (tm) {
         const int m = __ffsll((long long)tm) - 1;
         tm &= tm - 1;
+        HX_BOUND(m < N)
+#ifdef HX_CHECKED
+        {
+          // m's heap lies inside the warp's arena and holds at most its capacity
+          const int64_t cap = W->hcl[m] ? (int64_t)8 << W->hcl[m] : 0;
+          HX_BOUND(W->hoff[m] >= 0 && W->hoff[m] + cap <= a.arena_per_warp && W->hsize[m] <= cap &&
+                   W->cnt[m] <= c.inst_slots[m])
+        }
+#endif
         uint64_t* const sl = W->slot + c.slot_base[m];
         const int ns = c.inst_slots[m];
         const unsigned pm = __ballot_sync(kFull, lane < npend && pend_m == m);
@@ -921,9 +973,11 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             rid = top.rid;
             svc = top.svc;
           }
+          HX_BOUND(rid >= 0 && rid < nc && cn < ns)
           start_call(sl, m, cn, rid, svc);
           ++cn;
         }
+        HX_STOP_IF_FAILED()
         if (lane == 0) W->cnt[m] = cn;
         set_key(m, cn ? sl[0] : kKeyInf);
       }

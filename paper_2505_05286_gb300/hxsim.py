@@ -20,10 +20,13 @@ import numpy as np
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libhxsim.so")
+# the same library built with every simulation-kernel index range-checked
+# (-DHX_CHECKED): a failed check is the per-simulation status HX_ERR_BOUNDS
+LIB_CHECKED_PATH = os.path.join(_PKG, "libhxsim_checked.so")
 HEADER = os.path.join(os.path.dirname(_PKG), "include", "hxsim.h")
 
 (HX_OK, HX_ERR_INVALID, HX_ERR_CUDA, HX_ERR_OOM, HX_ERR_CAPACITY, HX_ERR_STEP_LIMIT, HX_ERR_STATE,
- HX_ERR_INVARIANT, HX_SKIPPED) = range(9)
+ HX_ERR_INVARIANT, HX_SKIPPED, HX_ERR_BOUNDS) = range(10)
 OBJ_P95, OBJ_P95_SLO95 = 0, 1
 
 RESULT_DTYPE = np.dtype([("p95_us", "<i8"), ("makespan_us", "<i8"), ("events", "<i8"),
@@ -99,8 +102,19 @@ def declared_functions() -> list:
     return sorted(set(re.findall(r"^\s*(?:int|const char\s*\*)\s+(hx_\w+)\s*\(", text, re.M)))
 
 
+_lib_checked = None
+
+
+def load_checked():
+    """Load the bounds-checked build libhxsim_checked.so; raises if it has not been built."""
+    global _lib_checked
+    if _lib_checked is None:
+        _lib_checked = load(LIB_CHECKED_PATH)
+    return _lib_checked
+
+
 def load(path: Optional[str] = None):
-    """Load libhxsim.so; raises if it has not been built."""
+    """Load libhxsim.so (or the library at `path`); raises if it has not been built."""
     global _lib
     if _lib is not None and path is None:
         return _lib
@@ -233,12 +247,14 @@ class Sim:
 
     def __init__(self, traces, cluster, grid, record_sims: Sequence[int] = (), timing: bool = False,
                  max_resident_warps: int = 0, force_generic: bool = False, subset: Optional[Sequence[int]] = None,
-                 checked: bool = False, arena_entries: int = 0):
+                 checked: bool = False, arena_entries: int = 0, bounds_checked: bool = False):
         """`subset`: run only these simulations (index trace * P + point); the
         others report HX_SKIPPED.  `checked`: also check the scheduler's
         invariants after every event (per-sim status HX_ERR_INVARIANT).
-        `arena_entries` (testing) caps each warp's local-queue arena."""
-        self.lib = load()
+        `arena_entries` (testing) caps each warp's local-queue arena.
+        `bounds_checked`: run on the bounds-checked build of the library
+        (per-sim status HX_ERR_BOUNDS if an index check fails)."""
+        self.lib = load_checked() if bounds_checked else load()
         self.n_traces = len(traces)
         self.n_points = int(grid.alpha_fp.shape[0])
         self.n_calls = [int(t.prompt.shape[0]) for t in traces]

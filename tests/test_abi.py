@@ -28,6 +28,13 @@ def test_exports_every_declared_function(lib):
         assert hasattr(lib, n), f"{n} declared in include/hxsim.h but not exported"
 
 
+def test_bounds_checked_build_exports_the_same_functions(lib):
+    chk = H.load_checked()
+    for n in H.declared_functions():
+        assert hasattr(chk, n), f"{n} missing from the bounds-checked build"
+    assert os.path.getsize(H.LIB_CHECKED_PATH) > 0 and chk is not lib
+
+
 _PROBE = r"""
 #include <stdio.h>
 #include <stddef.h>
