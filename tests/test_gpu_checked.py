@@ -32,7 +32,7 @@ def checked_sim(wl, **kw):
 def test_hand_cases_checked(name):
     tr, cl, exp = cases.hand_case(name)
     wl = W.Workload(name, [tr], cl, cases.grid_from_points([exp["point"]]), W.OBJ_P95)
-    sim = checked_sim(wl, record=[0])
+    sim = checked_sim(wl, record_sims=[0])
     r = sim.results()[0]
     assert r["status"] == H.HX_OK
     assert sim.records(0)["start"].tolist() == exp["start"]
@@ -44,7 +44,7 @@ def test_hand_cases_checked(name):
 @pytest.mark.parametrize("seed", range(24))
 def test_random_workloads_checked(seed, lean):
     wl = cases.random_workload(seed, lean=lean)
-    sim = checked_sim(wl, record=[] if lean else [wl.n_sims - 1])
+    sim = checked_sim(wl, record_sims=[] if lean else [wl.n_sims - 1])
     assert sim.info()["generic_kernel"] == (0 if lean else 1)
     o, oe = oracle.run(wl, range(wl.n_sims), extra=True)
     g = sim.results()
