@@ -45,7 +45,13 @@ SM_COUNT_FALLBACK = 152
 
 WARP_INST_PER_EVENT = 300
 KERNEL_SRC = os.path.join(ROOT, "paper_2505_05286_gb300", "csrc", "hx_kernels.cu")
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "hx_sim_kernel_traffic.txt")
+# ncu figures of the simulation kernel, each file keyed to the kernel source's
+# SHA-256: DRAM traffic of one full ceiling launch (a one-pass capture of the
+# DRAM byte counters alone), and issue-slot use and instruction mix per
+# simulated call event (a multi-metric capture of a small case that still
+# fills the GPU: 64 traces x 2000 queries x 1024 points)
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "hx_sim_kernel_ceiling_dram.txt")
+COUNTERS_FILE = os.path.join(ROOT, "profiles", "hx_sim_kernel_small_counters.txt")
 
 
 # grid-wide policy overrides (Sec. 5.1's ablations and baselines): local queue, dispatch
@@ -82,12 +88,12 @@ def _is_ceiling(args) -> bool:
             and args.alpha == "all" and args.policy == "grid")
 
 
-def _ncu_figures():
-    """Figures of the committed ncu captures of the simulation kernel on the
-    ceiling workload; {} when the kernel source changed since the capture."""
+def _ncu_figures(path=COUNTERS_FILE):
+    """key=value figures of a committed ncu capture of the simulation kernel;
+    {} when the kernel source changed since the capture."""
     import hashlib
     try:
-        kv = dict(line.strip().split("=", 1) for line in open(TRAFFIC_FILE)
+        kv = dict(line.strip().split("=", 1) for line in open(path)
                   if "=" in line and not line.startswith("#"))
         with open(KERNEL_SRC, "rb") as f:
             sha = hashlib.sha256(f.read()).hexdigest()
@@ -98,13 +104,68 @@ def _ncu_figures():
 
 def _traffic_per_launch(n_sims: int):
     """DRAM bytes (read + write) of one simulation-kernel launch on the
-    ceiling workload from the committed ncu capture, scaled to this launch's
-    simulations; None when the kernel source changed since the capture."""
-    kv = _ncu_figures()
+    ceiling workload from the committed full-size capture; None when the
+    kernel source changed since the capture."""
+    kv = _ncu_figures(TRAFFIC_FILE)
     try:
         return float(kv["dram_bytes_per_launch"]) * n_sims / float(kv["sims_per_launch"])
     except (KeyError, ValueError):
         return None
+
+
+def summarize_ncu(csv_path: str, bench_json: str, kind: str, command: str) -> str:
+    """key=value summary of an ncu CSV (--csv --log-file) of the simulation
+    kernel, per launch, with the kernel source's SHA-256; `bench_json` is the
+    bench line of the same command run without ncu (events and simulations
+    per launch).  kind: "ceiling" (DRAM bytes of a full launch) or "small"
+    (issue-slot use and instruction mix per simulated call event)."""
+    import csv
+    import hashlib
+    vals = {}
+    launches = set()
+    with open(csv_path) as f:
+        rows = [r for r in csv.reader(f) if r]
+    hdr = next(r for r in rows if r[0] == "ID")
+    for r in rows[rows.index(hdr) + 1:]:
+        d = dict(zip(hdr, r))
+        if "hx_sim_kernel" not in d.get("Kernel Name", ""):
+            continue
+        launches.add(d["ID"])
+        vals.setdefault(d["Metric Name"], []).append(float(d["Metric Value"].replace(",", "")))
+    n = len(launches)
+    per = {k: sum(v) / n for k, v in vals.items()}
+    line = json.loads(open(bench_json).read().strip().splitlines()[-1])
+    ev = float(line["roofline"]["events_per_launch"])
+    with open(KERNEL_SRC, "rb") as f:
+        sha = hashlib.sha256(f.read()).hexdigest()
+    out = [f"# ncu capture of hx_sim_kernel ({kind}), mean over {n} captured launch(es)",
+           f"# workload: {line['config']['workload']}, {line['config']['sims']} simulations, "
+           f"{int(ev)} simulated call events per launch",
+           f"# command: {command}", f"kernel_sha256={sha}", f"sims_per_launch={line['config']['sims']}",
+           f"events_per_launch={int(ev)}", f"kernel_ns={per.get('gpu__time_duration.sum', 0):.0f}"]
+    if "dram__bytes_read.sum" in per:
+        rd, wr = per["dram__bytes_read.sum"], per.get("dram__bytes_write.sum", 0.0)
+        out += [f"dram_read_bytes_per_launch={rd:.0f}", f"dram_write_bytes_per_launch={wr:.0f}",
+                f"dram_bytes_per_launch={rd + wr:.0f}"]
+    if kind == "small" and "smsp__inst_executed.sum" in per:
+        inst = per["smsp__inst_executed.sum"]
+        out += [f"issue_active_frac={per['smsp__issue_active.sum'] / per['smsp__cycles_active.sum']:.4f}",
+                f"warp_inst_per_event={inst / ev:.2f}",
+                f"threads_per_inst={per['smsp__thread_inst_executed.sum'] / inst:.2f}"]
+        for pipe in ("alu", "fma", "lsu", "cbu", "uniform", "adu", "xu"):
+            k = f"sm__inst_executed_pipe_{pipe}.sum"
+            if k in per:
+                out.append(f"{pipe}_inst_per_event={per[k] / ev:.2f}")
+        for op, name in (("branch", "branch"), ("shared_ld", "shared_load"), ("shared_st", "shared_store"),
+                         ("global_ld", "global_load"), ("global_st", "global_store"), ("local_ld", "local_load")):
+            k = f"sm__sass_inst_executed_op_{op}.sum"
+            if k in per:
+                out.append(f"{name}_inst_per_event={per[k] / ev:.2f}")
+        for k, name in (("l1tex__t_sector_hit_rate.pct", "l1_hit_pct"), ("lts__t_sector_hit_rate.pct", "l2_hit_pct"),
+                        ("smsp__warps_active.avg.per_cycle_active", "warps_active_per_scheduler")):
+            if k in per:
+                out.append(f"{name}={per[k]:.2f}")
+    return "\n".join(out) + "\n"
 
 
 def _peaks():
@@ -345,9 +406,12 @@ def run_gpu(args):
     # has seen every query arrive, so arrivals = completed queries)
     arrivals_per_step = int(res["n_done"].sum())
     all_events_rate = (events_per_step + arrivals_per_step) * world * args.steps / (t_ms / 1000.0)
-    prep_ms = float(np.median([x[0] for x in sim_ms]))
-    kern_ms = float(np.median([x[1] for x in sim_ms]))
-    best_ms = float(np.median([x[2] for x in sim_ms]))
+    # mean over the timed steps (each step's kernels lie inside that step, so the
+    # mean never exceeds ms_per_step); the median beside it
+    prep_ms = float(np.mean([x[0] for x in sim_ms]))
+    kern_ms = float(np.mean([x[1] for x in sim_ms]))
+    best_ms = float(np.mean([x[2] for x in sim_ms]))
+    kern_ms_median = float(np.median([x[1] for x in sim_ms]))
 
     # end to end through the C ABI from pinned host buffers: upload, run, read back
     e2e_steps = 1
@@ -394,9 +458,10 @@ def run_gpu(args):
     if _is_ceiling(args):
         # issue-slot use and executed instructions per event from the committed ncu capture
         kv = _ncu_figures()
-        for key in ("issue_active_frac", "warp_inst_per_event", "threads_per_inst"):
+        for key in ("issue_active_frac", "warp_inst_per_event", "threads_per_inst", "alu_inst_per_event",
+                    "fma_inst_per_event", "lsu_inst_per_event", "branch_inst_per_event"):
             if key in kv:
-                roofline["ncu_" + key] = float(kv[key])
+                roofline["ncu_small_case_" + key] = float(kv[key])
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic",
@@ -408,7 +473,8 @@ def run_gpu(args):
                               f"inputs fit in L2 ({n_calls * 64 / 2**20:.1f} MiB of call records), not flushed"),
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "resident_warps": info["resident_warps"], "blocks": info["blocks"]},
-            "kernels_ms": {"prep": prep_ms, "simulate": kern_ms, "best": best_ms},
+            "kernels_ms": {"prep": prep_ms, "simulate": kern_ms, "best": best_ms, "simulate_median": kern_ms_median,
+                           "over_steps": len(sim_ms)},
             "best_point": {"global_point": best[0], "sum_p95_us": best[1], "sum_slo_met": best[2]},
             "roofline": roofline, "clocks": clocks, "gpu_launches": 3 * args.steps,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
@@ -442,7 +508,15 @@ def main():
                     help="index of workloads.RECIPES or a key of workloads.EXTRA (default: the ceiling workload)")
     ap.add_argument("--policy", default="grid", choices=["grid"] + sorted(POLICIES),
                     help="one local-queue / dispatch policy on every grid point (default: the recipe's own)")
+    ap.add_argument("--summarize-ncu", nargs=3, metavar=("CSV", "BENCH_JSON", "KIND"), default=None,
+                    help="write the key=value summary of an ncu CSV of the simulation kernel (KIND: ceiling or "
+                         "small) to stdout; --ncu-command gives the command it came from")
+    ap.add_argument("--ncu-command", default="")
     args = ap.parse_args()
+    if args.summarize_ncu:
+        csv_path, bench_json, kind = args.summarize_ncu
+        sys.stdout.write(summarize_ncu(csv_path, bench_json, kind, args.ncu_command))
+        return
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -254,7 +254,7 @@ __device__ __noinline__ void digest_flush(WarpShared* W, int n, int lane) {
 }
 
 __device__ __forceinline__ void digest_push(WarpShared* W, int& dn, int64_t t, uint32_t tag, int lane) {
-  if (lane == 0) W->dterm[dn] = make_longlong2(t, (long long)tag);
+  W->dterm[dn] = make_longlong2(t, (long long)tag);  // every lane writes the same pair
   if (++dn == 16) {
     digest_flush(W, 16, lane);
     dn = 0;
@@ -470,9 +470,12 @@ __device__ __noinline__ int2 push_pop(WarpShared* W, const CallRec* rec, int64_t
 // All lanes: a query's evaluation call finished at `now` (Sec. 4.3's metrics).
 __device__ __forceinline__ void finish_query(WarpShared* W, int& dn, int32_t qid, int64_t now, int64_t arrival,
                                             int64_t deadline, int lane) {
-  if (lane == 0) {
-    W->slo_met += now <= deadline ? 1 : 0;
-    W->n_done++;
+  {
+    // every lane reads the counters, then every lane writes the same new values
+    const int32_t slo = W->slo_met + (now <= deadline ? 1 : 0), nd = W->n_done + 1;
+    __syncwarp();
+    W->slo_met = slo;
+    W->n_done = nd;
     W->makespan = now;
   }
   digest_push(W, dn, now, query_tag(qid), lane);
@@ -711,11 +714,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     };
 
     auto set_key = [&](int m, uint64_t nk) {
-      if (lane == (m & 31)) {
-        // an empty instance (nk all ones) maps to a key at or above kNoEvent
-        const uint64_t kk = ((nk >> 24) << 7) | (uint64_t)m;
-        if (m < 32) k0 = kk; else k1 = kk;
-      }
+      // an empty instance (nk all ones) maps to a key at or above kNoEvent
+      const uint64_t kk = ((nk >> 24) << 7) | (uint64_t)m;
+      k0 = lane == m ? kk : k0;
+      k1 = lane + 32 == m ? kk : k1;
     };
 
     for (;;) {
@@ -756,13 +758,14 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         __syncwarp();
         if (lane < cn) sl[lane] = nxt;
         if (faults && lane < cn) fl[lane] = fnxt;
-        if (lane == 0) W->cnt[m] = cn - 1;
+        W->cnt[m] = cn - 1;  // every lane writes the same count
         set_key(m, head);
-        if (lane == (m & 31)) {
-          W->q[m] -= est_m;
+        {
+          const int64_t qm = W->q[m];
+          if (lane == (m & 31)) W->q[m] = qm - est_m;
           const bool stale = W->rewards != 0;
-          if (m < 32) dirty0 = stale;
-          else dirty1 = stale;
+          dirty0 = lane == m ? stale : dirty0;
+          dirty1 = lane + 32 == m ? stale : dirty1;
         }
         // the freed slot needs a batch boundary only if requests wait for it
         if (hs_m > 0) touched |= 1ull << m;
@@ -778,7 +781,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         } else if (stg == HX_STAGE_S) {
           const int k = (tail.w >> 16) & 0xff;
           HX_BOUND(k >= 1 && k <= HX_MAX_K && rid + k < nc)
-          if (lane == 0) W->chains[qid] = (uint8_t)k;
+          W->chains[qid] = (uint8_t)k;  // every lane writes the same byte
           rel_first = rid + 1;
           rel_count = k;
         } else if (stg == HX_STAGE_E) {
@@ -812,7 +815,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             uint8_t* const chains = W->chains;
             const int left = chains[qid] - 1;
             __syncwarp();
-            if (lane == 0) chains[qid] = (uint8_t)left;
+            chains[qid] = (uint8_t)left;  // every lane writes the same byte
             rel_first = ~nx;
             rel_count = left == 0 ? 1 : 0;
           }
@@ -875,11 +878,12 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         // the winner's costs, from the lane that owns it
         const int64_t est_m = __shfl_sync(kFull, m < 32 ? e0 : e1, m & 31);
         const int svc_m = __shfl_sync(kFull, m < 32 ? v0 : v1, m & 31);
-        if (lane == (m & 31)) {
-          W->q[m] += est_m;
+        {
+          const int64_t qm = W->q[m];
+          if (lane == (m & 31)) W->q[m] = qm + est_m;
           const bool stale = W->rewards != 0;
-          if (m < 32) dirty0 = stale;
-          else dirty1 = stale;
+          dirty0 = lane == m ? stale : dirty0;
+          dirty1 = lane + 32 == m ? stale : dirty1;
         }
         if (kGeneric) {
           const int recj = W->recj;
@@ -900,20 +904,16 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           const int cn = W->cnt[m];
           if (W->hsize[m] == 0 && cn + (rel_count - jr) <= c.inst_slots[m]) {
             start_call(sl, m, cn, rid, svc_m);
-            if (lane == 0) W->cnt[m] = cn + 1;
+            W->cnt[m] = cn + 1;  // every lane writes the same count
             set_key(m, sl[0]);
             continue;
           }
         }
         // the local-queue key is formed only if the request has to wait
         HX_BOUND(npend < HX_MAX_K)
-        if (lane == npend) {
-          pend_m = m;
-        }
-        if (lane == 0) {
-          W->prs[npend] = make_int2(rid, svc_m);
-          W->pest[npend] = (int32_t)est_m;
-        }
+        pend_m = lane == npend ? m : pend_m;
+        W->prs[npend] = make_int2(rid, svc_m);  // every lane writes the same entry
+        W->pest[npend] = (int32_t)est_m;
         npend++;
         touched |= 1ull << m;
       }
@@ -969,7 +969,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
             __syncwarp();
             if (cn >= ns || n == 0) break;
             const HeapEnt top = heap_sift_warp(W->arena + W->hoff[m], n - 1, W->arena[W->hoff[m] + n - 1], lane);
-            if (lane == 0) W->hsize[m] = n - 1;
+            W->hsize[m] = n - 1;  // every lane writes the same size
             rid = top.rid;
             svc = top.svc;
           }
@@ -978,7 +978,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           ++cn;
         }
         HX_STOP_IF_FAILED()
-        if (lane == 0) W->cnt[m] = cn;
+        W->cnt[m] = cn;  // every lane writes the same count
         set_key(m, cn ? sl[0] : kKeyInf);
       }
       if (kGeneric && a.checked && status == HX_OK) {
