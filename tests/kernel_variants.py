@@ -3,9 +3,12 @@ library and timed against it on the same workload, each required to give
 bit-identical results.  This is how the alternatives the design notes
 mention were measured (GPU only).
 
-    python -m tests.kernel_variants prefetch [--traces 64] [--reps 3] [--out FILE]
+    python -m tests.kernel_variants FAMILY [--traces 64] [--reps 3] [--out FILE]
 
-Variants `prefetch`:
+Family `occupancy`: 8 or 6 resident 4-warp blocks per SM instead of 7 (the
+register budget follows), and the digest summed per lane in a register.
+
+Family `prefetch`:
   arrival_l1 / arrival_l2  at a query's arrival, prefetch its call records
                            (up to 10 records, 5 lines of 128 bytes) into L1 / L2;
   start_l1 / start_l2      when a request is dispatched, prefetch the records
@@ -49,14 +52,60 @@ _START = ("""        HX_BOUND(rid < nc)
             asm volatile("prefetch.global.LVL [%0];" ::"l"(pa));
         }""")
 
+# Each lane keeps the sum of the digest terms it hashes in a register; the
+# warp adds the 32 partial sums once, when the simulation ends, instead of a
+# shuffle reduction at every 16-term flush.
+_DIGEST_LANES = [
+    ("""__device__ __noinline__ void digest_flush(WarpShared* W, int n, int lane) {
+  __syncwarp();
+  const longlong2 e = W->dterm[lane < n ? lane : 0];
+  uint64_t y = lane < n ? digest_term((uint64_t)e.x, (uint64_t)e.y) : 0ull;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) y += __shfl_xor_sync(kFull, y, o);
+  if (lane == 0) W->digest += y;
+  __syncwarp();
+}""", """__device__ __noinline__ uint64_t digest_flush(WarpShared* W, int n, int lane) {
+  __syncwarp();
+  const longlong2 e = W->dterm[lane < n ? lane : 0];
+  const uint64_t y = lane < n ? digest_term((uint64_t)e.x, (uint64_t)e.y) : 0ull;
+  __syncwarp();
+  return y;
+}"""),
+    ("""__device__ __forceinline__ void digest_push(WarpShared* W, int& dn, int64_t t, uint32_t tag, int lane) {""",
+     """__device__ __forceinline__ void digest_push(WarpShared* W, int& dn, uint64_t& dacc, int64_t t, uint32_t tag,
+                                            int lane) {"""),
+    ("""    digest_flush(W, 16, lane);
+    dn = 0;""", """    dacc += digest_flush(W, 16, lane);
+    dn = 0;"""),
+    ("""__device__ __forceinline__ void finish_query(WarpShared* W, int& dn, int32_t qid,""",
+     """__device__ __forceinline__ void finish_query(WarpShared* W, int& dn, uint64_t& dacc, int32_t qid,"""),
+    ("""  digest_push(W, dn, now, query_tag(qid), lane);""", """  digest_push(W, dn, dacc, now, query_tag(qid), lane);"""),
+    ("""    int dn = 0;  // digest terms waiting in W->dterm""",
+     """    int dn = 0;  // digest terms waiting in W->dterm
+    uint64_t dacc = 0;  // this lane's share of the digest"""),
+    ("""      digest_push(W, dn, now, call_tag(rid, m), lane);""", """      digest_push(W, dn, dacc, now, call_tag(rid, m), lane);"""),
+    ("""          finish_query(W, dn, qid, now, arr, dl, lane);""", """          finish_query(W, dn, dacc, qid, now, arr, dl, lane);"""),
+    ("""    digest_flush(W, dn, lane);
+""", """    dacc += digest_flush(W, dn, lane);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) dacc += __shfl_xor_sync(kFull, dacc, o);
+    W->digest = dacc;
+    __syncwarp();
+"""),
+]
+
 VARIANTS = {
     "prefetch": {f"{w}_{lvl.lower()}": [(e[0], e[1].replace("LVL", lvl))]
                  for w, e in (("arrival", _ARRIVAL), ("start", _START)) for lvl in ("L1", "L2")},
+    # resident blocks per SM the register allocation aims at (7 by default), and the digest in registers
+    "occupancy": {"blocks8": ([], ["-DHX_SIM_MIN_BLOCKS=8"]), "blocks6": ([], ["-DHX_SIM_MIN_BLOCKS=6"]),
+                  "digest_lanes": (_DIGEST_LANES, [])},
 }
 
 
-def make_variant(name, edits):
-    """Copy the library sources, apply the edits to hx_kernels.cu, build a .so."""
+def make_variant(name, edits, flags=()):
+    """Copy the library sources, apply the edits to hx_kernels.cu, build a .so
+    (extra nvcc flags for hx_kernels.cu)."""
     d = os.path.join(OUT, name)
     shutil.rmtree(d, ignore_errors=True)
     shutil.copytree(CSRC, os.path.join(d, "csrc"))
@@ -70,7 +119,9 @@ def make_variant(name, edits):
     objs = []
     for src in ("hx_kernels.cu", "hx_api.cu"):
         o = os.path.join(d, src.replace(".cu", ".o"))
-        subprocess.check_call(NVCC + ["-I", os.path.join(d, "csrc"), "-c", os.path.join(d, "csrc", src), "-o", o])
+        extra = list(flags) if src == "hx_kernels.cu" else []
+        subprocess.check_call(NVCC + ["-I", os.path.join(d, "csrc"), *extra, "-c", os.path.join(d, "csrc", src),
+                                      "-o", o])
         objs.append(o)
     lib = os.path.join(d, "libhxsim.so")
     subprocess.check_call(NVCC[:3] + ["-shared", "-o", lib] + objs)
@@ -118,8 +169,9 @@ def main(argv=None):
     out = {"workload": f"{wl.name} cut to {args.traces} traces", "sims": wl.n_sims, "library_ms": base_ms,
            "library_all_ms": base_all, "variants": {}}
     print("library", base_ms, base_all, flush=True)
-    for name, edits in VARIANTS[args.family].items():
-        ms, all_ms, r = time_lib(make_variant(name, edits), wl, args.reps)
+    for name, spec in VARIANTS[args.family].items():
+        edits, flags = spec if isinstance(spec, tuple) else (spec, [])
+        ms, all_ms, r = time_lib(make_variant(name, edits, flags), wl, args.reps)
         same = all(np.array_equal(r[f], base[f]) for f in fields)
         out["variants"][name] = {"ms": ms, "all_ms": all_ms, "same_results": same, "speedup": base_ms / ms}
         print(name, ms, all_ms, same, round(base_ms / ms, 4), flush=True)
