@@ -126,6 +126,22 @@ def summarize_ncu(csv_path: str, bench_json: str, kind: str, command: str) -> st
     with open(csv_path) as f:
         rows = [r for r in csv.reader(f) if r]
     hdr = next(r for r in rows if r[0] == "ID")
+    if kind == "launches":
+        # every captured launch: per kernel its launches, total time and share
+        per_k = {}
+        for r in rows[rows.index(hdr) + 1:]:
+            d = dict(zip(hdr, r))
+            if d.get("Metric Name") == "gpu__time_duration.sum":
+                name = d["Kernel Name"].split("(")[0]
+                t = per_k.setdefault(name, [0, 0.0])
+                t[0] += 1
+                t[1] += float(d["Metric Value"].replace(",", "")) / 1e6
+        tot = sum(v[1] for v in per_k.values())
+        out = [f"# ncu launch list (gpu__time_duration.sum), command: {command}",
+               "| kernel | launches | total ms | share |", "|---|---|---|---|"]
+        for name, (n, ms) in sorted(per_k.items(), key=lambda kv: -kv[1][1]):
+            out.append(f"| {name} | {n} | {ms:.1f} | {100 * ms / tot:.3f} % |")
+        return "\n".join(out) + "\n"
     for r in rows[rows.index(hdr) + 1:]:
         d = dict(zip(hdr, r))
         if "hx_sim_kernel" not in d.get("Kernel Name", ""):
@@ -509,8 +525,8 @@ def main():
     ap.add_argument("--policy", default="grid", choices=["grid"] + sorted(POLICIES),
                     help="one local-queue / dispatch policy on every grid point (default: the recipe's own)")
     ap.add_argument("--summarize-ncu", nargs=3, metavar=("CSV", "BENCH_JSON", "KIND"), default=None,
-                    help="write the key=value summary of an ncu CSV of the simulation kernel (KIND: ceiling or "
-                         "small) to stdout; --ncu-command gives the command it came from")
+                    help="write the summary of an ncu CSV to stdout (KIND: ceiling or small: key=value figures of the "
+                         "simulation kernel; launches: the launch list); --ncu-command gives the command")
     ap.add_argument("--ncu-command", default="")
     args = ap.parse_args()
     if args.summarize_ncu:
