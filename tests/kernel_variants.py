@@ -5,6 +5,10 @@ mention were measured (GPU only).
 
     python -m tests.kernel_variants FAMILY [--traces 64] [--reps 3] [--out FILE]
 
+Family `micro`: the event key formed with one shift and a mask; the
+simulation's "rewards used" flag and its beta, beta as a float and 1 - alpha
+kept in registers instead of re-read from shared memory.
+
 Family `occupancy`: 8 or 6 resident 4-warp blocks per SM instead of 7 (the
 register budget follows), and the digest summed per lane in a register.
 
@@ -94,7 +98,42 @@ _DIGEST_LANES = [
 """),
 ]
 
+# Micro changes of the hot loop.
+_KEY_SHIFT = [("""      const uint64_t kk = ((nk >> 24) << 7) | (uint64_t)m;""",
+               """      const uint64_t kk = ((nk >> 17) & ~0x7Full) | (uint64_t)m;""")]
+_REWARDS_REG = [("""    const int32_t oma32 = W->one_minus_a;""",
+                 """    const int32_t oma32 = W->one_minus_a;
+    const bool rewards_on = W->rewards != 0;"""),
+                ("""          const bool stale = W->rewards != 0;
+          dirty0 = lane == m ? stale : dirty0;
+          dirty1 = lane + 32 == m ? stale : dirty1;
+        }
+        // the freed slot""", """          const bool stale = rewards_on;
+          dirty0 = lane == m ? stale : dirty0;
+          dirty1 = lane + 32 == m ? stale : dirty1;
+        }
+        // the freed slot"""),
+                ("""          const bool stale = W->rewards != 0;
+          dirty0 = lane == m ? stale : dirty0;
+          dirty1 = lane + 32 == m ? stale : dirty1;
+        }
+        if (kGeneric) {""", """          const bool stale = rewards_on;
+          dirty0 = lane == m ? stale : dirty0;
+          dirty1 = lane + 32 == m ? stale : dirty1;
+        }
+        if (kGeneric) {""")]
+_BETA_REGS = [("""    const int32_t oma32 = W->one_minus_a;""",
+               """    const int32_t oma32 = W->one_minus_a;
+    const uint64_t beta_r = (uint64_t)W->beta;
+    const float betaf_r = W->betaf;"""),
+              ("""        const uint64_t beta = (uint64_t)W->beta;""", """        const uint64_t beta = beta_r;"""),
+              ("""rj ? W->betaf : 0.0f""", """rj ? betaf_r : 0.0f"""),
+              ("""              (int64_t)W->one_minus_a * (res < (uint64_t)kRewardCap""",
+               """              (int64_t)oma32 * (res < (uint64_t)kRewardCap""")]
+
 VARIANTS = {
+    "micro": {"key_shift": _KEY_SHIFT, "rewards_reg": _REWARDS_REG, "beta_regs": _BETA_REGS,
+              "all_three": _KEY_SHIFT + _REWARDS_REG + _BETA_REGS},
     "prefetch": {f"{w}_{lvl.lower()}": [(e[0], e[1].replace("LVL", lvl))]
                  for w, e in (("arrival", _ARRIVAL), ("start", _START)) for lvl in ("L1", "L2")},
     # resident blocks per SM the register allocation aims at (7 by default), and the digest in registers
