@@ -642,6 +642,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     // (1 - alpha) * reward per instance; instances past N score far below any
     // real one (|alpha * est| < 2^52), so the argmax needs no validity test
     const int32_t oma32 = W->one_minus_a;
+    // rewards carry weight (alpha < 1 with workload-balanced dispatch): kept in
+    // a predicate register rather than re-read at every queue-cost change
+    const bool rewards_on = W->rewards != 0;
     const int64_t orew_idle = (int64_t)oma32 * reward_of(W->beta, 0);
     int64_t orew0 = valid0 ? orew_idle : -(int64_t(1) << 62);
     int64_t orew1 = valid1 ? orew_idle : -(int64_t(1) << 62);
@@ -763,7 +766,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         {
           const int64_t qm = W->q[m];
           if (lane == (m & 31)) W->q[m] = qm - est_m;
-          const bool stale = W->rewards != 0;
+          const bool stale = rewards_on;
           dirty0 = lane == m ? stale : dirty0;
           dirty1 = lane + 32 == m ? stale : dirty1;
         }
@@ -881,7 +884,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         {
           const int64_t qm = W->q[m];
           if (lane == (m & 31)) W->q[m] = qm + est_m;
-          const bool stale = W->rewards != 0;
+          const bool stale = rewards_on;
           dirty0 = lane == m ? stale : dirty0;
           dirty1 = lane + 32 == m ? stale : dirty1;
         }

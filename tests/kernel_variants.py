@@ -6,8 +6,8 @@ mention were measured (GPU only).
     python -m tests.kernel_variants FAMILY [--traces 64] [--reps 3] [--out FILE]
 
 Family `micro`: the event key formed with one shift and a mask; the
-simulation's "rewards used" flag and its beta, beta as a float and 1 - alpha
-kept in registers instead of re-read from shared memory.
+simulation's beta, beta as a float and 1 - alpha, or its alpha, kept in
+registers instead of re-read from shared memory.
 
 Family `occupancy`: 8 or 6 resident 4-warp blocks per SM instead of 7 (the
 register budget follows), and the digest summed per lane in a register.
@@ -131,9 +131,16 @@ _BETA_REGS = [("""    const int32_t oma32 = W->one_minus_a;""",
               ("""              (int64_t)W->one_minus_a * (res < (uint64_t)kRewardCap""",
                """              (int64_t)oma32 * (res < (uint64_t)kRewardCap""")]
 
+_A_REG = [("""    const bool rewards_on = W->rewards != 0;""",
+           """    const bool rewards_on = W->rewards != 0;
+    const int32_t alpha_r = W->A;"""),
+          ("""          const int32_t A = W->A;""", """          const int32_t A = alpha_r;""")]
+
 VARIANTS = {
-    "micro": {"key_shift": _KEY_SHIFT, "rewards_reg": _REWARDS_REG, "beta_regs": _BETA_REGS,
-              "all_three": _KEY_SHIFT + _REWARDS_REG + _BETA_REGS},
+    # measured on 64 ceiling traces: key_shift 1.000, beta_regs 0.992 (the
+    # "rewards used" flag in a predicate register gave 1.013 and is now in the
+    # library); alpha_reg is measured against the library that includes it
+    "micro": {"key_shift": _KEY_SHIFT, "beta_regs": _BETA_REGS, "alpha_reg": _A_REG},
     "prefetch": {f"{w}_{lvl.lower()}": [(e[0], e[1].replace("LVL", lvl))]
                  for w, e in (("arrival", _ARRIVAL), ("start", _START)) for lvl in ("L1", "L2")},
     # resident blocks per SM the register allocation aims at (7 by default), and the digest in registers
