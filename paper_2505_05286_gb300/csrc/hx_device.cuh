@@ -144,6 +144,8 @@ struct SimArgs {
 // order, so the next completion on it is always its first slot.
 struct WarpShared {
   int64_t q[HX_MAX_INST];       // t_queue: Eq. comp summed over requests dispatched and unfinished
+  uint64_t ekey[HX_MAX_INST];   // next completion event key per instance
+  int64_t orew[HX_MAX_INST];    // cached (1 - alpha) * reward per instance (its owner lane's)
   int32_t hoff[HX_MAX_INST];    // local queue: heap offset in the arena
   int32_t hsize[HX_MAX_INST];   //              heap size
   uint8_t cnt[HX_MAX_INST];     // running calls (the first cnt of the instance's slot keys)

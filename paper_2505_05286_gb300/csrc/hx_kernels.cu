@@ -494,6 +494,7 @@ __device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, i
 
 }  // namespace
 
+// Resident blocks per SM the register allocation aims for (4 warps each).
 #ifndef HX_SIM_MIN_BLOCKS
 #define HX_SIM_MIN_BLOCKS 7
 #endif
@@ -518,7 +519,7 @@ __device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, i
 #define HX_BOUND(cond)
 #define HX_STOP_IF_FAILED()
 #endif
-// Resident blocks per SM the register allocation aims for (4 warps each).
+
 template <bool kGeneric>
 __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -636,7 +637,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     __syncwarp();
 
     // this lane's instances: queue cost, cached reward and its staleness, event keys
-    // (t_queue of instance m lives in W->q[m], touched only by its owner lane)
+    // (t_queue and the next completion key of instance m live in W->q[m] and
+    // W->ekey[m], each change stored alike by every lane; its cached reward in
+    // W->orew[m], written and read by the owner lane alone; shared memory
+    // rather than registers leaves the allocator room)
     W->q[m0] = 0;
     W->q[m1] = 0;
     // (1 - alpha) * reward per instance; instances past N score far below any
@@ -646,10 +650,11 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     // a predicate register rather than re-read at every queue-cost change
     const bool rewards_on = W->rewards != 0;
     const int64_t orew_idle = (int64_t)oma32 * reward_of(W->beta, 0);
-    int64_t orew0 = valid0 ? orew_idle : -(int64_t(1) << 62);
-    int64_t orew1 = valid1 ? orew_idle : -(int64_t(1) << 62);
+    W->orew[m0] = valid0 ? orew_idle : -(int64_t(1) << 62);
+    W->orew[m1] = valid1 ? orew_idle : -(int64_t(1) << 62);
     bool dirty0 = false, dirty1 = false;
-    uint64_t k0 = kKeyInf, k1 = kKeyInf;
+    W->ekey[m0] = kKeyInf;
+    W->ekey[m1] = kKeyInf;
     // this event's dispatches, entry j on lane j
     int pend_m = -1;
 
@@ -718,13 +723,12 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
 
     auto set_key = [&](int m, uint64_t nk) {
       // an empty instance (nk all ones) maps to a key at or above kNoEvent
-      const uint64_t kk = ((nk >> 24) << 7) | (uint64_t)m;
-      k0 = lane == m ? kk : k0;
-      k1 = lane + 32 == m ? kk : k1;
+      W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key
     };
 
     for (;;) {
       HX_STOP_IF_FAILED()
+      const uint64_t k0 = W->ekey[m0], k1 = W->ekey[m1];
       const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
       const uint64_t akey = W->akey;
       if (ck >= kNoEvent && akey == kKeyInf) break;
@@ -764,8 +768,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         W->cnt[m] = cn - 1;  // every lane writes the same count
         set_key(m, head);
         {
-          const int64_t qm = W->q[m];
-          if (lane == (m & 31)) W->q[m] = qm - est_m;
+          W->q[m] = W->q[m] - est_m;  // every lane stores the same value
           const bool stale = rewards_on;
           dirty0 = lane == m ? stale : dirty0;
           dirty1 = lane + 32 == m ? stale : dirty1;
@@ -854,8 +857,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           const uint64_t res = udiv_trial_f(rj ? beta : 0ull, rj ? W->betaf : 0.0f, (rj && q > 1) ? (uint64_t)q : 1ull);
           const int64_t orew =
               (int64_t)W->one_minus_a * (res < (uint64_t)kRewardCap ? (int64_t)res : kRewardCap);
-          if (dirty0) { orew0 = orew; dirty0 = false; }
-          else if (dirty1) { orew1 = orew; dirty1 = false; }
+          if (rj) W->orew[dirty0 ? m0 : m1] = orew;
+          if (dirty0) dirty0 = false;
+          else dirty1 = false;
         }
         int m;
         // a re-issued request avoids the instance it timed out on
@@ -867,8 +871,8 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           if (lane == 0) W->rr = (m + 1 == N) ? 0 : m + 1;
         } else {
           const int32_t A = W->A;
-          int64_t s0 = orew0 - (int64_t)A * e0;
-          int64_t s1 = orew1 - (int64_t)A * e1;
+          int64_t s0 = W->orew[m0] - (int64_t)A * e0;
+          int64_t s1 = W->orew[m1] - (int64_t)A * e1;
           if (kGeneric && excl >= 0) {
             if (m0 == excl) s0 = INT64_MIN;
             if (m1 == excl) s1 = INT64_MIN;
@@ -882,8 +886,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         const int64_t est_m = __shfl_sync(kFull, m < 32 ? e0 : e1, m & 31);
         const int svc_m = __shfl_sync(kFull, m < 32 ? v0 : v1, m & 31);
         {
-          const int64_t qm = W->q[m];
-          if (lane == (m & 31)) W->q[m] = qm + est_m;
+          W->q[m] = W->q[m] + est_m;  // every lane stores the same value
           const bool stale = rewards_on;
           dirty0 = lane == m ? stale : dirty0;
           dirty1 = lane + 32 == m ? stale : dirty1;

@@ -5,6 +5,15 @@ mention were measured (GPU only).
 
     python -m tests.kernel_variants FAMILY [--traces 64] [--reps 3] [--out FILE]
 
+Family `state`: the instance of each pending dispatch kept in shared memory
+instead of on the entry's lane; the lane's instance types re-read at each
+dispatch from the kernel parameters or from a shared copy; 8 resident
+blocks per SM.
+
+Family `misc`: the next arrival in the next-event minimum; the request id
+of each instance's next completion kept beside its key; the heap sift, or
+the queue push helpers, inlined.
+
 Family `micro`: the event key formed with one shift and a mask; the
 simulation's beta, beta as a float and 1 - alpha, or its alpha, kept in
 registers instead of re-read from shared memory.
@@ -99,8 +108,8 @@ _DIGEST_LANES = [
 ]
 
 # Micro changes of the hot loop.
-_KEY_SHIFT = [("""      const uint64_t kk = ((nk >> 24) << 7) | (uint64_t)m;""",
-               """      const uint64_t kk = ((nk >> 17) & ~0x7Full) | (uint64_t)m;""")]
+_KEY_SHIFT = [("""      W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key""",
+               """      W->ekey[m] = ((nk >> 17) & ~0x7Full) | (uint64_t)m;  // every lane stores the same key""")]
 _REWARDS_REG = [("""    const int32_t oma32 = W->one_minus_a;""",
                  """    const int32_t oma32 = W->one_minus_a;
     const bool rewards_on = W->rewards != 0;"""),
@@ -136,10 +145,77 @@ _A_REG = [("""    const bool rewards_on = W->rewards != 0;""",
     const int32_t alpha_r = W->A;"""),
           ("""          const int32_t A = W->A;""", """          const int32_t A = alpha_r;""")]
 
+_HDR = "hx_device.cuh"
+# The instance each of this event's dispatches went to, in shared memory
+# beside the entry instead of on the entry's lane; the lane's two instance
+# types read from the kernel's parameters at each dispatch.
+_PEND_SMEM = [(_HDR, """  int32_t pest[HX_MAX_K];""", """  int32_t pest[HX_MAX_K];
+  int32_t pendm[HX_MAX_K];"""),
+              ("""    // this event's dispatches, entry j on lane j
+    int pend_m = -1;
+""", ""),
+              ("""        pend_m = lane == npend ? m : pend_m;""",
+               """        W->pendm[npend] = m;  // every lane writes the same entry"""),
+              ("""        const unsigned pm = __ballot_sync(kFull, lane < npend && pend_m == m);""",
+               """        const unsigned pm = __ballot_sync(kFull, lane < npend && W->pendm[lane < npend ? lane : 0] == m);""")]
+_TY_PARAM = [("""  const int ty0 = valid0 ? c.inst_type[m0] : 0;
+  const int ty1 = valid1 ? c.inst_type[m1] : 0;
+""", ""),
+             ("""        const int e0 = r->est[ty0], e1 = r->est[ty1];""",
+              """        const int ty0 = c.inst_type[m0], ty1 = c.inst_type[m1];  // 0 past the cluster's instances
+        const int e0 = r->est[ty0], e1 = r->est[ty1];""")]
+# ... or from a per-warp shared copy filled once per kernel.
+_TY_SMEM = [(_HDR, """  uint8_t hcl[HX_MAX_INST];""", """  uint8_t hcl[HX_MAX_INST];
+  uint8_t ity[HX_MAX_INST];      // instance types (0 past the cluster's instances)"""),
+            ("""  const int ty0 = valid0 ? c.inst_type[m0] : 0;
+  const int ty1 = valid1 ? c.inst_type[m1] : 0;
+""", """  W->ity[m0] = c.inst_type[m0];
+  W->ity[m1] = c.inst_type[m1];
+"""),
+            ("""        const int e0 = r->est[ty0], e1 = r->est[ty1];""",
+             """        const int ty0 = W->ity[m0], ty1 = W->ity[m1];
+        const int e0 = r->est[ty0], e1 = r->est[ty1];""")]
+_B8 = ["-DHX_SIM_MIN_BLOCKS=8"]
+
+# The next arrival joins the next-event minimum on lane 0 (at equal times a
+# completion, tag < 64, still goes first).
+_ARR_IN_MIN = [("""      const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
+      const uint64_t akey = W->akey;
+      if (ck >= kNoEvent && akey == kKeyInf) break;""", """      const uint64_t akey = W->akey;
+      const uint64_t k01 = k0 < k1 ? k0 : k1;
+      const uint64_t ck = warp_min_u64(lane == 0 && akey < k01 ? akey : k01);
+      if (ck >= kNoEvent) break;"""),
+               ("""      if (ck < akey) {
+        // completion on instance m""", """      if ((ck & 127ull) != kArrivalTag) {
+        // completion on instance m""")]
+# The request id of each instance's next completion kept beside its event
+# key, so that the finishing call's record load waits on one shared load
+# rather than on the slot base and the first slot.
+_ERID = [(_HDR, """  uint64_t ekey[HX_MAX_INST];   // next completion event key per instance""",
+          """  uint64_t ekey[HX_MAX_INST];   // next completion event key per instance
+  int32_t erid[HX_MAX_INST];    // its request id"""),
+         ("""      W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key""",
+          """      W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key
+      W->erid[m] = (int32_t)(nk & 0xffffffull);"""),
+         ("""        const int32_t rid = (int32_t)(sl[0] & 0xffffffull);""", """        const int32_t rid = W->erid[m];""")]
+_INLINE_SIFT = [("""__device__ __noinline__ HeapEnt heap_sift_warp(""", """__device__ __forceinline__ HeapEnt heap_sift_warp(""")]
+_INLINE_PUSH = [("""__device__ __noinline__ int push_pending(""", """__device__ __forceinline__ int push_pending("""),
+                ("""__device__ __noinline__ int2 push_pop(""", """__device__ __forceinline__ int2 push_pop(""")]
+
 VARIANTS = {
+    # measured on 64 ceiling traces: against the library that kept the event
+    # keys and rewards in registers, both in shared memory 1.0135 (keys alone
+    # 1.002, rewards alone 0.996); against that, t_queue stored by every lane
+    # 1.0097 (both now in the library), pend_smem 0.990, ty_param 0.914,
+    # ty_smem 0.993, both 0.993, blocks8 0.958
+    "state": {"pend_smem": (_PEND_SMEM, []), "ty_param": (_TY_PARAM, []), "ty_smem": (_TY_SMEM, []),
+              "pend_ty_smem": (_PEND_SMEM + _TY_SMEM, []), "blocks8": ([], _B8)},
     # measured on 64 ceiling traces: key_shift 1.000, beta_regs 0.992 (the
     # "rewards used" flag in a predicate register gave 1.013 and is now in the
     # library); alpha_reg is measured against the library that includes it
+    "misc": {"arr_in_min": (_ARR_IN_MIN, []), "erid": (_ERID, []), "inline_sift": (_INLINE_SIFT, []),
+             "inline_push": (_INLINE_PUSH, []), "inline_both": (_INLINE_SIFT + _INLINE_PUSH, []),
+             "arr_erid": (_ARR_IN_MIN + _ERID, [])},
     "micro": {"key_shift": _KEY_SHIFT, "beta_regs": _BETA_REGS, "alpha_reg": _A_REG},
     "prefetch": {f"{w}_{lvl.lower()}": [(e[0], e[1].replace("LVL", lvl))]
                  for w, e in (("arrival", _ARRIVAL), ("start", _START)) for lvl in ("L1", "L2")},
@@ -150,18 +226,19 @@ VARIANTS = {
 
 
 def make_variant(name, edits, flags=()):
-    """Copy the library sources, apply the edits to hx_kernels.cu, build a .so
-    (extra nvcc flags for hx_kernels.cu)."""
+    """Copy the library sources, apply the edits ((anchor, replacement) in
+    hx_kernels.cu, or (file, anchor, replacement)), build a .so (extra nvcc
+    flags for hx_kernels.cu)."""
     d = os.path.join(OUT, name)
     shutil.rmtree(d, ignore_errors=True)
     shutil.copytree(CSRC, os.path.join(d, "csrc"))
-    p = os.path.join(d, "csrc", "hx_kernels.cu")
-    s = open(p).read()
-    for a, b in edits:
+    for e in edits:
+        f, a, b = e if len(e) == 3 else ("hx_kernels.cu", *e)
+        p = os.path.join(d, "csrc", f)
+        s = open(p).read()
         if a not in s:
-            raise RuntimeError(f"variant {name}: anchor not found in hx_kernels.cu: {a[:60]!r}")
-        s = s.replace(a, b)
-    open(p, "w").write(s)
+            raise RuntimeError(f"variant {name}: anchor not found in {f}: {a[:60]!r}")
+        open(p, "w").write(s.replace(a, b))
     objs = []
     for src in ("hx_kernels.cu", "hx_api.cu"):
         o = os.path.join(d, src.replace(".cu", ".o"))
