@@ -145,6 +145,7 @@ struct SimArgs {
 struct WarpShared {
   int64_t q[HX_MAX_INST];       // t_queue: Eq. comp summed over requests dispatched and unfinished
   uint64_t ekey[HX_MAX_INST];   // next completion event key per instance
+  int32_t erid[HX_MAX_INST];    // its request id
   int64_t orew[HX_MAX_INST];    // cached (1 - alpha) * reward per instance (its owner lane's)
   int32_t hoff[HX_MAX_INST];    // local queue: heap offset in the arena
   int32_t hsize[HX_MAX_INST];   //              heap size

@@ -289,7 +289,7 @@ __device__ __forceinline__ void heap_push(HeapEnt* h, int n, long long key, int 
 // `sink` takes its place, sinking to its level; the heap then holds m
 // entries (m = n - 1 and sink = the last entry: a pop; m = n and sink = a new
 // entry: a replace).  Every lane gets the old top.
-__device__ __noinline__ HeapEnt heap_sift_warp(HeapEnt* h, int m, HeapEnt sink, int lane) {
+__device__ __forceinline__ HeapEnt heap_sift_warp(HeapEnt* h, int m, HeapEnt sink, int lane) {
   const HeapEnt top = h[0];
   int i = 0;
   for (;;) {
@@ -412,7 +412,7 @@ __device__ __forceinline__ long long pending_key(const WarpShared* W, const Call
 
 // The instance's new requests (pending entries, bits of pm) join its local
 // queue, their keys formed one per lane.
-__device__ __noinline__ int push_pending(WarpShared* W, const CallRec* rec, int64_t now, int lpol,
+__device__ __forceinline__ int push_pending(WarpShared* W, const CallRec* rec, int64_t now, int lpol,
                                         int64_t arena_per_warp, int m, unsigned pm, int lane) {
   const long long key = ((pm >> lane) & 1u) ? pending_key(W, rec, now, lpol, lane) : 0;
   HeapEnt* const arena = W->arena;
@@ -451,7 +451,7 @@ __device__ __noinline__ int push_pending(WarpShared* W, const CallRec* rec, int6
 // and a non-empty local queue: the more urgent of it and the queue's top
 // starts and the other waits, i.e. a push and a pop in one sift (the new
 // request replaces the top).  Returns the started (request id, service time).
-__device__ __noinline__ int2 push_pop(WarpShared* W, const CallRec* rec, int64_t now, int lpol, int m, unsigned pm,
+__device__ __forceinline__ int2 push_pop(WarpShared* W, const CallRec* rec, int64_t now, int lpol, int m, unsigned pm,
                                      int lane) {
   const int j = __ffs(pm) - 1;
   const long long key = __shfl_sync(kFull, lane == j ? pending_key(W, rec, now, lpol, j) : 0, j);
@@ -496,7 +496,7 @@ __device__ __noinline__ void log_dispatch(const SimArgs& a, int recj, int rid, i
 
 // Resident blocks per SM the register allocation aims for (4 warps each).
 #ifndef HX_SIM_MIN_BLOCKS
-#define HX_SIM_MIN_BLOCKS 7
+#define HX_SIM_MIN_BLOCKS 8
 #endif
 
 // Bounds-checked build (-DHX_CHECKED): before every shared- or global-memory
@@ -724,6 +724,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     auto set_key = [&](int m, uint64_t nk) {
       // an empty instance (nk all ones) maps to a key at or above kNoEvent
       W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key
+      W->erid[m] = (int32_t)(nk & 0xffffffull);
     };
 
     for (;;) {
@@ -748,8 +749,9 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         uint64_t* const sl = W->slot + c.slot_base[m];
         const int cn = W->cnt[m];
         HX_BOUND(cn >= 1 && cn <= c.inst_slots[m] && c.slot_base[m] + cn <= c.total_slots)
-        // the finishing call heads m's sorted slots
-        const int32_t rid = (int32_t)(sl[0] & 0xffffffull);
+        // the finishing call heads m's sorted slots; its id is kept beside
+        // m's event key, so that its record load need not wait for the slot
+        const int32_t rid = W->erid[m];
         HX_BOUND(rid < nc)
         // the finished call's record: issued now, used after the slot shift
         const CallRec* r = rec + rid;

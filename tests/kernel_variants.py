@@ -7,18 +7,16 @@ mention were measured (GPU only).
 
 Family `state`: the instance of each pending dispatch kept in shared memory
 instead of on the entry's lane; the lane's instance types re-read at each
-dispatch from the kernel parameters or from a shared copy; 8 resident
-blocks per SM.
+dispatch from the kernel parameters or from a shared copy.
 
-Family `misc`: the next arrival in the next-event minimum; the request id
-of each instance's next completion kept beside its key; the heap sift, or
-the queue push helpers, inlined.
+Family `misc`: the next arrival in the next-event minimum; the digest
+flush, or the top-K insert, inlined.
 
 Family `micro`: the event key formed with one shift and a mask; the
 simulation's beta, beta as a float and 1 - alpha, or its alpha, kept in
 registers instead of re-read from shared memory.
 
-Family `occupancy`: 8 or 6 resident 4-warp blocks per SM instead of 7 (the
+Family `occupancy`: 7 or 6 resident 4-warp blocks per SM instead of 8 (the
 register budget follows), and the digest summed per lane in a register.
 
 Family `prefetch`:
@@ -175,7 +173,6 @@ _TY_SMEM = [(_HDR, """  uint8_t hcl[HX_MAX_INST];""", """  uint8_t hcl[HX_MAX_IN
             ("""        const int e0 = r->est[ty0], e1 = r->est[ty1];""",
              """        const int ty0 = W->ity[m0], ty1 = W->ity[m1];
         const int e0 = r->est[ty0], e1 = r->est[ty1];""")]
-_B8 = ["-DHX_SIM_MIN_BLOCKS=8"]
 
 # The next arrival joins the next-event minimum on lane 0 (at equal times a
 # completion, tag < 64, still goes first).
@@ -188,39 +185,37 @@ _ARR_IN_MIN = [("""      const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
                ("""      if (ck < akey) {
         // completion on instance m""", """      if ((ck & 127ull) != kArrivalTag) {
         // completion on instance m""")]
-# The request id of each instance's next completion kept beside its event
-# key, so that the finishing call's record load waits on one shared load
-# rather than on the slot base and the first slot.
-_ERID = [(_HDR, """  uint64_t ekey[HX_MAX_INST];   // next completion event key per instance""",
-          """  uint64_t ekey[HX_MAX_INST];   // next completion event key per instance
-  int32_t erid[HX_MAX_INST];    // its request id"""),
-         ("""      W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key""",
-          """      W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key
-      W->erid[m] = (int32_t)(nk & 0xffffffull);"""),
-         ("""        const int32_t rid = (int32_t)(sl[0] & 0xffffffull);""", """        const int32_t rid = W->erid[m];""")]
-_INLINE_SIFT = [("""__device__ __noinline__ HeapEnt heap_sift_warp(""", """__device__ __forceinline__ HeapEnt heap_sift_warp(""")]
-_INLINE_PUSH = [("""__device__ __noinline__ int push_pending(""", """__device__ __forceinline__ int push_pending("""),
-                ("""__device__ __noinline__ int2 push_pop(""", """__device__ __forceinline__ int2 push_pop(""")]
+_INLINE_DIGEST = [("""__device__ __noinline__ void digest_flush(""", """__device__ __forceinline__ void digest_flush(""")]
+_INLINE_TOPK = [("""__device__ __noinline__ void topk_insert_warp(""", """__device__ __forceinline__ void topk_insert_warp(""")]
 
 VARIANTS = {
     # measured on 64 ceiling traces: against the library that kept the event
     # keys and rewards in registers, both in shared memory 1.0135 (keys alone
     # 1.002, rewards alone 0.996); against that, t_queue stored by every lane
     # 1.0097 (both now in the library), pend_smem 0.990, ty_param 0.914,
-    # ty_smem 0.993, both 0.993, blocks8 0.958
+    # ty_smem 0.993, both 0.993, 8 blocks per SM 0.958 (64 registers, spills);
+    # with the heap helpers inlined (no spills left at 72 registers): 8 blocks
+    # per SM 1.028 (no spills at 64; now the library's), pend_smem 0.998,
+    # ty_param 0.920, ty_smem 0.994, both 0.997
     "state": {"pend_smem": (_PEND_SMEM, []), "ty_param": (_TY_PARAM, []), "ty_smem": (_TY_SMEM, []),
-              "pend_ty_smem": (_PEND_SMEM + _TY_SMEM, []), "blocks8": ([], _B8)},
+              "pend_ty_smem": (_PEND_SMEM + _TY_SMEM, [])},
     # measured on 64 ceiling traces: key_shift 1.000, beta_regs 0.992 (the
     # "rewards used" flag in a predicate register gave 1.013 and is now in the
     # library); alpha_reg is measured against the library that includes it
-    "misc": {"arr_in_min": (_ARR_IN_MIN, []), "erid": (_ERID, []), "inline_sift": (_INLINE_SIFT, []),
-             "inline_push": (_INLINE_PUSH, []), "inline_both": (_INLINE_SIFT + _INLINE_PUSH, []),
-             "arr_erid": (_ARR_IN_MIN + _ERID, [])},
+    # measured on 64 ceiling traces: arr_in_min 0.988, erid 1.004, the heap
+    # sift inlined 1.005, the queue push helpers 1.007, both 1.014 (now in
+    # the library), arr_in_min with erid 1.000; on the library with the
+    # inlined helpers: arr_in_min 0.997, erid 1.005, inline_digest 0.998,
+    # inline_topk 0.996, erid_topk 1.011; at 8 blocks per SM: arr_in_min
+    # 0.996, erid 1.006 (now in the library), inline_digest 0.998,
+    # inline_topk 1.006, erid_topk 1.006
+    "misc": {"arr_in_min": (_ARR_IN_MIN, []), "inline_digest": (_INLINE_DIGEST, []),
+             "inline_topk": (_INLINE_TOPK, [])},
     "micro": {"key_shift": _KEY_SHIFT, "beta_regs": _BETA_REGS, "alpha_reg": _A_REG},
     "prefetch": {f"{w}_{lvl.lower()}": [(e[0], e[1].replace("LVL", lvl))]
                  for w, e in (("arrival", _ARRIVAL), ("start", _START)) for lvl in ("L1", "L2")},
-    # resident blocks per SM the register allocation aims at (7 by default), and the digest in registers
-    "occupancy": {"blocks8": ([], ["-DHX_SIM_MIN_BLOCKS=8"]), "blocks6": ([], ["-DHX_SIM_MIN_BLOCKS=6"]),
+    # resident blocks per SM the register allocation aims at (8 by default), and the digest in registers
+    "occupancy": {"blocks7": ([], ["-DHX_SIM_MIN_BLOCKS=7"]), "blocks6": ([], ["-DHX_SIM_MIN_BLOCKS=6"]),
                   "digest_lanes": (_DIGEST_LANES, [])},
 }
 
