@@ -900,8 +900,8 @@ int hx_sim_prep(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int3
   HX_CUDA(cudaMemcpy(recs.data(), h->d_rec + off, n_calls * sizeof(hx::CallRec), cudaMemcpyDeviceToHost));
   for (size_t j = 0; j < n_calls; ++j) {
     for (int ty = 0; ty < 4; ++ty) {
-      if (est) est[4 * j + ty] = recs[j].est[ty];
-      if (svc) svc[4 * j + ty] = recs[j].svc[ty];
+      if (est) est[4 * j + ty] = recs[j].ev[ty].x;
+      if (svc) svc[4 * j + ty] = recs[j].ev[ty].y;
     }
     if (tbar) tbar[j] = recs[j].tbar;
     if (deadline_us) deadline_us[j] = recs[j].deadline;

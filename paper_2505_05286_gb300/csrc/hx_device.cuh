@@ -32,8 +32,8 @@ constexpr int kFRows = 18;                // S, G/C with 0..15 corrections done,
 
 // One call as the simulator reads it: 64 bytes, 16-byte aligned.
 struct __align__(16) CallRec {
-  int32_t est[4];     // Eq. (comp) with the believed output length, per type
-  int32_t svc[4];     // the same with the true output length (service time)
+  int2 ev[4];         // per type: Eq. (comp) with the believed output length, and the
+                      // same with the true output length (service time)
   int64_t deadline;   // query arrival + T_slo
   int64_t arrival;    // query arrival
   int32_t tbar;       // mean of est over the instances

@@ -193,12 +193,10 @@ __global__ void __launch_bounds__(256) hx_prep_kernel(PrepArgs a, ClusterK c) {
       if (ty < T) {
         const int64_t pre = ceil_div_pos(p * kUsPerS, c.prefill[ty]);
         const int64_t es = pre + oe * (int64_t)c.decode[ty];
-        r.est[ty] = (int32_t)es;
-        r.svc[ty] = (int32_t)(pre + o * (int64_t)c.decode[ty]);
+        r.ev[ty] = make_int2((int32_t)es, (int32_t)(pre + o * (int64_t)c.decode[ty]));
         sum += es * c.cnt[ty];
       } else {
-        r.est[ty] = 0;
-        r.svc[ty] = 0;
+        r.ev[ty] = make_int2(0, 0);
       }
     }
     r.tbar = (int32_t)(sum / c.n_inst);
@@ -692,7 +690,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
           }
         }
         if (in_window && c.timeout_mult_fp > 0) {
-          const int64_t timeout = ((int64_t)rec[rid].est[c.inst_type[m]] * c.timeout_mult_fp) / kScale;
+          const int64_t timeout = ((int64_t)rec[rid].ev[c.inst_type[m]].x * c.timeout_mult_fp) / kScale;
           if (down || run > timeout) {
             fail = true;
             run = timeout;
@@ -756,7 +754,7 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         // the finished call's record: issued now, used after the slot shift
         const CallRec* r = rec + rid;
         const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
-        const int64_t est_m = r->est[c.inst_type[m]];
+        const int64_t est_m = r->ev[c.inst_type[m]].x;
         const int hs_m = W->hsize[m];
         // remove it: the remaining keys move down one slot
         const uint64_t nxt = lane + 1 < cn ? sl[lane + 1] : kKeyInf;
@@ -848,8 +846,8 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
         HX_BOUND(rid < nc)
         const CallRec* r = rec + rid;
         // Eq. (comp) and the service time on this lane's two instances
-        const int e0 = r->est[ty0], e1 = r->est[ty1];
-        const int v0 = r->svc[ty0], v1 = r->svc[ty1];
+        const int2 ev0 = r->ev[ty0], ev1 = r->ev[ty1];
+        const int e0 = ev0.x, e1 = ev1.x, v0 = ev0.y, v1 = ev1.y;
         // SIMT division passes: each lane refreshes one stale reward of its
         // instances per pass (two passes at most)
         const uint64_t beta = (uint64_t)W->beta;

@@ -12,6 +12,9 @@ dispatch from the kernel parameters or from a shared copy.
 Family `misc`: the next arrival in the next-event minimum; the digest
 flush, or the top-K insert, inlined.
 
+Family `layout`: a lane's two event keys and two cached rewards adjacent in
+shared memory.
+
 Family `micro`: the event key formed with one shift and a mask; the
 simulation's beta, beta as a float and 1 - alpha, or its alpha, kept in
 registers instead of re-read from shared memory.
@@ -159,9 +162,9 @@ _PEND_SMEM = [(_HDR, """  int32_t pest[HX_MAX_K];""", """  int32_t pest[HX_MAX_K
 _TY_PARAM = [("""  const int ty0 = valid0 ? c.inst_type[m0] : 0;
   const int ty1 = valid1 ? c.inst_type[m1] : 0;
 """, ""),
-             ("""        const int e0 = r->est[ty0], e1 = r->est[ty1];""",
+             ("""        const int2 ev0 = r->ev[ty0], ev1 = r->ev[ty1];""",
               """        const int ty0 = c.inst_type[m0], ty1 = c.inst_type[m1];  // 0 past the cluster's instances
-        const int e0 = r->est[ty0], e1 = r->est[ty1];""")]
+        const int2 ev0 = r->ev[ty0], ev1 = r->ev[ty1];""")]
 # ... or from a per-warp shared copy filled once per kernel.
 _TY_SMEM = [(_HDR, """  uint8_t hcl[HX_MAX_INST];""", """  uint8_t hcl[HX_MAX_INST];
   uint8_t ity[HX_MAX_INST];      // instance types (0 past the cluster's instances)"""),
@@ -170,9 +173,9 @@ _TY_SMEM = [(_HDR, """  uint8_t hcl[HX_MAX_INST];""", """  uint8_t hcl[HX_MAX_IN
 """, """  W->ity[m0] = c.inst_type[m0];
   W->ity[m1] = c.inst_type[m1];
 """),
-            ("""        const int e0 = r->est[ty0], e1 = r->est[ty1];""",
+            ("""        const int2 ev0 = r->ev[ty0], ev1 = r->ev[ty1];""",
              """        const int ty0 = W->ity[m0], ty1 = W->ity[m1];
-        const int e0 = r->est[ty0], e1 = r->est[ty1];""")]
+        const int2 ev0 = r->ev[ty0], ev1 = r->ev[ty1];""")]
 
 # The next arrival joins the next-event minimum on lane 0 (at equal times a
 # completion, tag < 64, still goes first).
@@ -185,6 +188,27 @@ _ARR_IN_MIN = [("""      const uint64_t ck = warp_min_u64(k0 < k1 ? k0 : k1);
                ("""      if (ck < akey) {
         // completion on instance m""", """      if ((ck & 127ull) != kArrivalTag) {
         // completion on instance m""")]
+# A lane's two event keys, and its two cached rewards, adjacent in shared
+# memory: one 16-byte load each at the loop top and at the argmax.
+_PAIRS = [("""      W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key""",
+           """      W->ekey[((m & 31) << 1) | (m >> 5)] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane stores the same key"""),
+          ("""    W->ekey[m0] = kKeyInf;
+    W->ekey[m1] = kKeyInf;""", """    W->ekey[2 * lane] = kKeyInf;
+    W->ekey[2 * lane + 1] = kKeyInf;"""),
+          ("""      const uint64_t k0 = W->ekey[m0], k1 = W->ekey[m1];""",
+           """      const ulonglong2 kp = *reinterpret_cast<const ulonglong2*>(&W->ekey[2 * lane]);
+      const uint64_t k0 = kp.x, k1 = kp.y;"""),
+          ("""    W->orew[m0] = valid0 ? orew_idle : -(int64_t(1) << 62);
+    W->orew[m1] = valid1 ? orew_idle : -(int64_t(1) << 62);""",
+           """    W->orew[2 * lane] = valid0 ? orew_idle : -(int64_t(1) << 62);
+    W->orew[2 * lane + 1] = valid1 ? orew_idle : -(int64_t(1) << 62);"""),
+          ("""          if (rj) W->orew[dirty0 ? m0 : m1] = orew;""", """          if (rj) W->orew[2 * lane + (dirty0 ? 0 : 1)] = orew;"""),
+          ("""          int64_t s0 = W->orew[m0] - (int64_t)A * e0;
+          int64_t s1 = W->orew[m1] - (int64_t)A * e1;""",
+           """          const longlong2 op = *reinterpret_cast<const longlong2*>(&W->orew[2 * lane]);
+          int64_t s0 = op.x - (int64_t)A * e0;
+          int64_t s1 = op.y - (int64_t)A * e1;""")]
+
 _INLINE_DIGEST = [("""__device__ __noinline__ void digest_flush(""", """__device__ __forceinline__ void digest_flush(""")]
 _INLINE_TOPK = [("""__device__ __noinline__ void topk_insert_warp(""", """__device__ __forceinline__ void topk_insert_warp(""")]
 
@@ -211,6 +235,9 @@ VARIANTS = {
     # inline_topk 1.006, erid_topk 1.006
     "misc": {"arr_in_min": (_ARR_IN_MIN, []), "inline_digest": (_INLINE_DIGEST, []),
              "inline_topk": (_INLINE_TOPK, [])},
+    # measured on 64 ceiling traces: (est, svc) side by side in the call
+    # record 1.009 (now in the library), pairs 0.991, both 0.994
+    "layout": {"pairs": (_PAIRS, [])},
     "micro": {"key_shift": _KEY_SHIFT, "beta_regs": _BETA_REGS, "alpha_reg": _A_REG},
     "prefetch": {f"{w}_{lvl.lower()}": [(e[0], e[1].replace("LVL", lvl))]
                  for w, e in (("arrival", _ARRIVAL), ("start", _START)) for lvl in ("L1", "L2")},
