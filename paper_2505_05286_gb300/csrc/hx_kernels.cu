@@ -452,7 +452,7 @@ __device__ __forceinline__ int push_pending(WarpShared* W, const CallRec* rec, i
 __device__ __forceinline__ int2 push_pop(WarpShared* W, const CallRec* rec, int64_t now, int lpol, int m, unsigned pm,
                                      int lane) {
   const int j = __ffs(pm) - 1;
-  const long long key = __shfl_sync(kFull, lane == j ? pending_key(W, rec, now, lpol, j) : 0, j);
+  const long long key = pending_key(W, rec, now, lpol, j);  // the same on every lane
   const int2 rs = W->prs[j];
   HeapEnt* const h = W->arena + W->hoff[m];
   const HeapEnt top = h[0];

@@ -15,6 +15,9 @@ flush, or the top-K insert, inlined.
 Family `layout`: a lane's two event keys and two cached rewards adjacent in
 shared memory.
 
+Family `heap`: the heap sift's move-up test taken from the reduced maximum
+key.
+
 Family `micro`: the event key formed with one shift and a mask; the
 simulation's beta, beta as a float and 1 - alpha, or its alpha, kept in
 registers instead of re-read from shared memory.
@@ -209,6 +212,12 @@ _PAIRS = [("""      W->ekey[m] = ((nk >> 24) << 7) | (uint64_t)m;  // every lane
           int64_t s0 = op.x - (int64_t)A * e0;
           int64_t s1 = op.y - (int64_t)A * e1;""")]
 
+# Heap sift: whether the best child moves up is decided from the reduced
+# maximum key itself (the child's rid is shuffled only on a key tie).
+_SIFT_NOSHFL = [("""    if (!__shfl_sync(kFull, (int)ent_better(ck, cr, sink.key, sink.rid), b)) break;""",
+                 """    const long long kb = (long long)((((uint64_t)mh << 32) | ml) ^ 0x8000000000000000ull);
+    if (kb < sink.key || (kb == sink.key && __shfl_sync(kFull, cr, b) >= sink.rid)) break;""")]
+
 _INLINE_DIGEST = [("""__device__ __noinline__ void digest_flush(""", """__device__ __forceinline__ void digest_flush(""")]
 _INLINE_TOPK = [("""__device__ __noinline__ void topk_insert_warp(""", """__device__ __forceinline__ void topk_insert_warp(""")]
 
@@ -238,6 +247,10 @@ VARIANTS = {
     # measured on 64 ceiling traces: (est, svc) side by side in the call
     # record 1.009 (now in the library), pairs 0.991, both 0.994
     "layout": {"pairs": (_PAIRS, [])},
+    # measured on 64 ceiling traces: sift_noshfl 0.992, push_pop's key formed
+    # on every lane rather than on the entry's lane and shuffled 1.006 (now in
+    # the library), both 0.998, pend_smem 0.994
+    "heap": {"sift_noshfl": (_SIFT_NOSHFL, [])},
     "micro": {"key_shift": _KEY_SHIFT, "beta_regs": _BETA_REGS, "alpha_reg": _A_REG},
     "prefetch": {f"{w}_{lvl.lower()}": [(e[0], e[1].replace("LVL", lvl))]
                  for w, e in (("arrival", _ARRIVAL), ("start", _START)) for lvl in ("L1", "L2")},
