@@ -571,7 +571,10 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
       W->clk0 = clk0;
     }
 
+    // per-instance state that every lane reads later: written before the
+    // barrier below
     for (int m = lane; m < 64; m += 32) {
+      W->q[m] = 0;
       W->hoff[m] = 0;
       W->hcl[m] = 0;
       W->hsize[m] = 0;
@@ -634,15 +637,14 @@ __device__ __forceinline__ void sim_body(const SimArgs& a, const ClusterK& c) {
     }
     __syncwarp();
 
-    // this lane's instances: queue cost, cached reward and its staleness, event keys
-    // (t_queue and the next completion key of instance m live in W->q[m] and
-    // W->ekey[m], each change stored alike by every lane; its cached reward in
-    // W->orew[m], written and read by the owner lane alone; shared memory
-    // rather than registers leaves the allocator room)
-    W->q[m0] = 0;
-    W->q[m1] = 0;
-    // (1 - alpha) * reward per instance; instances past N score far below any
-    // real one (|alpha * est| < 2^52), so the argmax needs no validity test
+    // this lane's instances m0 = lane and m1 = lane + 32: t_queue in W->q[m]
+    // and the next completion's event key and request id in W->ekey[m] and
+    // W->erid[m] (every change stored alike by every lane; the owner reads
+    // the keys at the loop top), the cached (1 - alpha) * reward in
+    // W->orew[m] (the owner lane alone) and its staleness in dirty0 / dirty1;
+    // shared memory rather than registers leaves the allocator room.
+    // Instances past N start with a reward far below any real score
+    // (|alpha * est| < 2^52), so the argmax needs no validity test.
     const int32_t oma32 = W->one_minus_a;
     // rewards carry weight (alpha < 1 with workload-balanced dispatch): kept in
     // a predicate register rather than re-read at every queue-cost change

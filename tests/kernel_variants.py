@@ -18,6 +18,9 @@ shared memory.
 Family `heap`: the heap sift's move-up test taken from the reduced maximum
 key.
 
+Family `div`: the reward pass's division without its divergent early
+return; a warp barrier after each simulation's per-lane initial state.
+
 Family `micro`: the event key formed with one shift and a mask; the
 simulation's beta, beta as a float and 1 - alpha, or its alpha, kept in
 registers instead of re-read from shared memory.
@@ -218,6 +221,19 @@ _SIFT_NOSHFL = [("""    if (!__shfl_sync(kFull, (int)ent_better(ck, cr, sink.key
                  """    const long long kb = (long long)((((uint64_t)mh << 32) | ml) ^ 0x8000000000000000ull);
     if (kb < sink.key || (kb == sink.key && __shfl_sync(kFull, cr, b) >= sink.rid)) break;""")]
 
+# The reward pass without the divergent early return of the division: an
+# idle instance (t_queue <= 1) divides by 2^62 like an inactive lane and
+# takes beta by a select.
+_DIV_UNIFORM = [("""          const uint64_t res = udiv_trial_f(rj ? beta : 0ull, rj ? W->betaf : 0.0f, (rj && q > 1) ? (uint64_t)q : 1ull);""",
+                 """          const uint64_t res0 =
+              udiv_trial_f(rj ? beta : 0ull, rj ? W->betaf : 0.0f, (rj && q > 1) ? (uint64_t)q : (1ull << 62));
+          const uint64_t res = (rj && q <= 1) ? beta : res0;""")]
+# A warp barrier after each simulation's per-lane initial state.
+_SYNC_INIT = [("""    W->akey = nq > 0 ? (((uint64_t)a.arrival[qb] << 7) | kArrivalTag) : kKeyInf;
+""", """    W->akey = nq > 0 ? (((uint64_t)a.arrival[qb] << 7) | kArrivalTag) : kKeyInf;
+    __syncwarp();  // every lane's initial instance state is read by the others
+""")]
+
 _INLINE_DIGEST = [("""__device__ __noinline__ void digest_flush(""", """__device__ __forceinline__ void digest_flush(""")]
 _INLINE_TOPK = [("""__device__ __noinline__ void topk_insert_warp(""", """__device__ __forceinline__ void topk_insert_warp(""")]
 
@@ -251,6 +267,11 @@ VARIANTS = {
     # on every lane rather than on the entry's lane and shuffled 1.006 (now in
     # the library), both 0.998, pend_smem 0.994
     "heap": {"sift_noshfl": (_SIFT_NOSHFL, [])},
+    # measured on 64 ceiling traces (3 runs each, library 4127 / 4131 ms):
+    # sync_init 0.997, div_uniform 0.998, both 0.997 -- within the run-to-run
+    # spread; t_queue is now zeroed before the existing barrier instead
+    "div": {"sync_init": (_SYNC_INIT, []), "div_uniform": (_DIV_UNIFORM, []),
+            "div_sync": (_DIV_UNIFORM + _SYNC_INIT, [])},
     "micro": {"key_shift": _KEY_SHIFT, "beta_regs": _BETA_REGS, "alpha_reg": _A_REG},
     "prefetch": {f"{w}_{lvl.lower()}": [(e[0], e[1].replace("LVL", lvl))]
                  for w, e in (("arrival", _ARRIVAL), ("start", _START)) for lvl in ("L1", "L2")},
