@@ -50,6 +50,9 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2505_05286_gb300", "csrc", "hx_kernels.cu
 # DRAM byte counters alone), and issue-slot use and instruction mix per
 # simulated call event (a multi-metric capture of a small case that still
 # fills the GPU: 64 traces x 2000 queries x 1024 points)
+# hx_info.work_order: the order the kernel takes the simulations in
+WORK_ORDERS = {0: "trace-major, highest point first", 1: "the subset's",
+               2: "every trace's alpha = 1 points first, then trace-major"}
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "hx_sim_kernel_ceiling_dram.txt")
 COUNTERS_FILE = os.path.join(ROOT, "profiles", "hx_sim_kernel_small_counters.txt")
 
@@ -488,7 +491,8 @@ def run_gpu(args):
                               if n_calls * 64 > L2_BYTES else
                               f"inputs fit in L2 ({n_calls * 64 / 2**20:.1f} MiB of call records), not flushed"),
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                       "resident_warps": info["resident_warps"], "blocks": info["blocks"]},
+                       "resident_warps": info["resident_warps"], "blocks": info["blocks"],
+                       "work_order": WORK_ORDERS[info["work_order"]]},
             "kernels_ms": {"prep": prep_ms, "simulate": kern_ms, "best": best_ms, "simulate_median": kern_ms_median,
                            "over_steps": len(sim_ms)},
             "best_point": {"global_point": best[0], "sum_p95_us": best[1], "sum_slo_met": best[2]},

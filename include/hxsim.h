@@ -359,7 +359,12 @@ typedef struct hx_info {
   int32_t smem_per_block;
   int32_t generic_kernel;       /* 1: the kernel with logging and every policy; 0: the
                                    PQ + workload-balanced instantiation without logging */
-  int32_t reserved;
+  int32_t work_order;           /* order the simulations are taken in: 0 trace-major, highest
+                                   point first; 1 the caller's subset (likewise ordered);
+                                   2 every trace's workload-balanced alpha = 1 points first
+                                   (their long local queues make them the costliest), chosen
+                                   when the run is 1-4 waves of warps deep and every trace's
+                                   records fit in L2.  Results never depend on it. */
 } hx_info;
 
 int hx_sim_info(hx_sim* h, hx_info* out);

@@ -136,8 +136,9 @@ struct hx_sim {
   int64_t rec_stride = 0;
   int32_t* d_rec_map = nullptr;
   // run only these simulations, in work order (NULL: all of them)
-  int64_t* d_subset = nullptr;
+  int64_t* d_subset = nullptr;  // the work order when not the kernel's own (see work_order)
   int64_t n_work = 0;
+  int32_t work_order = 0;       // hx_info.work_order
   bool checked = false;
   int32_t* d_rec_inst = nullptr;
   int64_t* d_rec_enq = nullptr;
@@ -455,6 +456,34 @@ int order_subset(const hx_options* opt, int32_t n_traces, int32_t n_points, std:
   return HX_OK;
 }
 
+// Work order for a whole grid when it pays to change the default one.  The
+// kernel takes simulations trace-major (the warps on one trace share its
+// records in L2), highest point first within a trace.  A simulation whose
+// points dispatch workload-balanced at alpha = 1 sends every request to the
+// fastest instance and builds the longest local queue, so it costs more per
+// event than any other point.  When the run is only a few waves of warps
+// deep, trace-major order starts the last traces' such simulations in the
+// last wave, and they set the end of the run; if every trace's records fit
+// in L2 together, nothing is lost by starting all of them first.  Returns an
+// empty order when the default stands.  Results do not depend on the order.
+std::vector<int64_t> costliest_first(const hx_grid* grid, int32_t n_traces, int64_t n_calls, int64_t l2_bytes,
+                                     int64_t resident_warps) {
+  std::vector<int64_t> order;
+  const int32_t P = grid->n_points;
+  const int64_t n_sims = (int64_t)n_traces * P;
+  if (n_sims <= resident_warps || n_sims > 4 * resident_warps) return order;
+  if (n_calls * (int64_t)sizeof(hx::CallRec) > l2_bytes) return order;
+  std::vector<int32_t> hot, cold;
+  for (int32_t p = P - 1; p >= 0; --p)
+    (grid->alpha_fp[p] == hx::kScale && grid->dispatch_policy[p] == HX_DISPATCH_WB ? hot : cold).push_back(p);
+  if (hot.empty() || cold.empty()) return order;
+  order.reserve((size_t)n_sims);
+  for (const std::vector<int32_t>* part : {&hot, &cold})
+    for (int32_t t = 0; t < n_traces; ++t)
+      for (int32_t p : *part) order.push_back((int64_t)t * P + p);
+  return order;
+}
+
 }  // namespace
 
 extern "C" {
@@ -551,9 +580,6 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
       (rc = upload(h->d_lp, grid->local_policy, h->n_points, s0)) ||
       (rc = upload(h->d_dp, grid->dispatch_policy, h->n_points, s0)))
     return bail(rc);
-  if (!subset.empty() && ((rc = h->alloc(&h->d_subset, (int64_t)subset.size())) ||
-                          (rc = upload(h->d_subset, subset.data(), (int64_t)subset.size(), s0))))
-    return bail(rc);
 
   h->generic = needs_generic(grid, ck, opt && opt->n_record > 0, opt && opt->force_generic, h->checked);
   const void* kfn = h->generic ? (const void*)hx::hx_sim_kernel : (const void*)hx::hx_sim_kernel_lean;
@@ -573,6 +599,15 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   blocks = std::min<int64_t>(blocks, (h->n_sims + hx::kWarpsPerBlock - 1) / hx::kWarpsPerBlock);
   h->blocks = (int)std::max<int64_t>(blocks, 1);
   h->resident_warps = h->blocks * hx::kWarpsPerBlock;
+  // the simulations' order: the caller's subset, else possibly the costliest first
+  h->work_order = subset.empty() ? 0 : 1;
+  if (subset.empty()) {
+    subset = costliest_first(grid, n_traces, h->n_c, (int64_t)prop.l2CacheSize, h->resident_warps);
+    if (!subset.empty()) h->work_order = 2;
+  }
+  if (!subset.empty() && ((rc = h->alloc(&h->d_subset, (int64_t)subset.size())) ||
+                          (rc = upload(h->d_subset, subset.data(), (int64_t)subset.size(), s0))))
+    return bail(rc);
   // heap arena: doubling regions of 16, 32, ... entries per instance total at
   // most 4 * (requests ever queued) + 16 * instances
   h->arena_per_warp = 4 * (int64_t)h->max_nc + 16 * HX_MAX_INST;
@@ -677,7 +712,7 @@ int hx_sim_run(hx_sim* h, void* stream) {
   pa.work_counter = h->d_counter;
   pa.skip_results = h->d_results;
   pa.skip_extras = h->d_extras;
-  pa.n_skip = h->d_subset ? h->n_sims : 0;
+  pa.n_skip = h->n_work < h->n_sims ? h->n_sims : 0;
 
   hx::SimArgs sa;
   sa.rec = h->d_rec;
@@ -966,7 +1001,7 @@ int hx_sim_info(hx_sim* h, hx_info* out) {
   out->blocks = h->blocks;
   out->smem_per_block = h->smem_per_block;
   out->generic_kernel = h->generic ? 1 : 0;
-  out->reserved = 0;
+  out->work_order = h->work_order;
   return HX_OK;
 }
 

@@ -89,7 +89,7 @@ class hx_info(ctypes.Structure):
                 ("device_bytes", ctypes.c_int64), ("resident_warps", ctypes.c_int32),
                 ("warps_per_block", ctypes.c_int32), ("blocks", ctypes.c_int32),
                 ("smem_per_block", ctypes.c_int32), ("generic_kernel", ctypes.c_int32),
-                ("reserved", ctypes.c_int32)]
+                ("work_order", ctypes.c_int32)]
 
 
 _lib = None

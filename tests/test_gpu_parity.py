@@ -608,6 +608,24 @@ def test_subset_runs_only_the_listed_simulations(generic):
     sim.close()
 
 
+@pytest.mark.parametrize("generic", [False, True])
+def test_costliest_first_order_changes_no_result(generic):
+    # 4 traces x 64 points on 64 resident warps: four waves, records far
+    # below L2, so every trace's workload-balanced alpha = 1 points go first
+    wl = W.make_workload(1, n_traces=4, n_queries=300)
+    sim = gpu(wl, max_resident_warps=64, force_generic=generic)
+    assert sim.info()["work_order"] == 2
+    r = sim.results()
+    assert_same(r, oracle_results(wl, range(wl.n_sims)), "costliest first")
+    check_best(sim, wl, r)
+    sim.close()
+    # one wave: the default order; a subset: its own
+    for kw, order in (({}, 0), ({"subset": list(range(0, wl.n_sims, 3)), "max_resident_warps": 64}, 1)):
+        s2 = gpu(wl, force_generic=generic, **kw)
+        assert s2.info()["work_order"] == order
+        s2.close()
+
+
 @pytest.mark.parametrize("name,nt,nq", [(1, 2, 300), ("faulty", 1, 1400), ("competing-50", 1, 300)])
 def test_checked_mode_changes_nothing(name, nt, nq):
     """With the per-event invariant checks on (generic kernel), every
