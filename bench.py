@@ -52,7 +52,8 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2505_05286_gb300", "csrc", "hx_kernels.cu
 # fills the GPU: 64 traces x 2000 queries x 1024 points)
 # hx_info.work_order: the order the kernel takes the simulations in
 WORK_ORDERS = {0: "trace-major, highest point first", 1: "the subset's",
-               2: "every trace's alpha = 1 points first, then trace-major"}
+               2: "every trace's alpha = 1 points first, then trace-major",
+               3: "trace-major; the last two waves' traces with their alpha = 1 points first"}
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "hx_sim_kernel_ceiling_dram.txt")
 COUNTERS_FILE = os.path.join(ROOT, "profiles", "hx_sim_kernel_small_counters.txt")
 

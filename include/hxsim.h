@@ -364,7 +364,9 @@ typedef struct hx_info {
                                    2 every trace's workload-balanced alpha = 1 points first
                                    (their long local queues make them the costliest), chosen
                                    when the run is 1-4 waves of warps deep and every trace's
-                                   records fit in L2.  Results never depend on it. */
+                                   records fit in L2; 3 trace-major, but the traces of about
+                                   the last two waves take their alpha = 1 points first
+                                   (deeper runs).  Results never depend on it. */
 } hx_info;
 
 int hx_sim_info(hx_sim* h, hx_info* out);

@@ -461,27 +461,36 @@ int order_subset(const hx_options* opt, int32_t n_traces, int32_t n_points, std:
 // records in L2), highest point first within a trace.  A simulation whose
 // points dispatch workload-balanced at alpha = 1 sends every request to the
 // fastest instance and builds the longest local queue, so it costs more per
-// event than any other point.  When the run is only a few waves of warps
-// deep, trace-major order starts the last traces' such simulations in the
-// last wave, and they set the end of the run; if every trace's records fit
-// in L2 together, nothing is lost by starting all of them first.  Returns an
-// empty order when the default stands.  Results do not depend on the order.
-std::vector<int64_t> costliest_first(const hx_grid* grid, int32_t n_traces, int64_t n_calls, int64_t l2_bytes,
-                                     int64_t resident_warps) {
-  std::vector<int64_t> order;
+// event than any other point, and trace-major order starts the last traces'
+// such simulations in the last wave, where they set the end of the run.  If
+// the run is at most four waves of warps deep and every trace's records fit
+// in L2 together, all traces' alpha = 1 points go first (hx_info.work_order
+// 2); otherwise the traces of about the last two waves take theirs first,
+// the others staying trace-major (3).  *order is left empty, and 0 returned,
+// when the default stands.  Results do not depend on the order.
+int costliest_first(const hx_grid* grid, int32_t n_traces, int64_t n_calls, int64_t l2_bytes,
+                    int64_t resident_warps, std::vector<int64_t>* order) {
+  order->clear();
   const int32_t P = grid->n_points;
   const int64_t n_sims = (int64_t)n_traces * P;
-  if (n_sims <= resident_warps || n_sims > 4 * resident_warps) return order;
-  if (n_calls * (int64_t)sizeof(hx::CallRec) > l2_bytes) return order;
+  if (n_sims <= resident_warps) return 0;
   std::vector<int32_t> hot, cold;
   for (int32_t p = P - 1; p >= 0; --p)
     (grid->alpha_fp[p] == hx::kScale && grid->dispatch_policy[p] == HX_DISPATCH_WB ? hot : cold).push_back(p);
-  if (hot.empty() || cold.empty()) return order;
-  order.reserve((size_t)n_sims);
+  if (hot.empty() || cold.empty()) return 0;
+  int32_t t0 = 0;  // traces before t0 keep the default order
+  if (n_sims > 4 * resident_warps || n_calls * (int64_t)sizeof(hx::CallRec) > l2_bytes) {
+    const int64_t k = (2 * resident_warps + P - 1) / P;
+    if (k >= n_traces) return 0;
+    t0 = n_traces - (int32_t)k;
+  }
+  order->reserve((size_t)n_sims);
+  for (int32_t t = 0; t < t0; ++t)
+    for (int32_t p = P - 1; p >= 0; --p) order->push_back((int64_t)t * P + p);
   for (const std::vector<int32_t>* part : {&hot, &cold})
-    for (int32_t t = 0; t < n_traces; ++t)
-      for (int32_t p : *part) order.push_back((int64_t)t * P + p);
-  return order;
+    for (int32_t t = t0; t < n_traces; ++t)
+      for (int32_t p : *part) order->push_back((int64_t)t * P + p);
+  return t0 == 0 ? 2 : 3;
 }
 
 }  // namespace
@@ -600,11 +609,9 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   h->blocks = (int)std::max<int64_t>(blocks, 1);
   h->resident_warps = h->blocks * hx::kWarpsPerBlock;
   // the simulations' order: the caller's subset, else possibly the costliest first
-  h->work_order = subset.empty() ? 0 : 1;
-  if (subset.empty()) {
-    subset = costliest_first(grid, n_traces, h->n_c, (int64_t)prop.l2CacheSize, h->resident_warps);
-    if (!subset.empty()) h->work_order = 2;
-  }
+  h->work_order = subset.empty()
+                      ? costliest_first(grid, n_traces, h->n_c, (int64_t)prop.l2CacheSize, h->resident_warps, &subset)
+                      : 1;
   if (!subset.empty() && ((rc = h->alloc(&h->d_subset, (int64_t)subset.size())) ||
                           (rc = upload(h->d_subset, subset.data(), (int64_t)subset.size(), s0))))
     return bail(rc);

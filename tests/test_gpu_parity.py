@@ -619,10 +619,14 @@ def test_costliest_first_order_changes_no_result(generic):
     assert_same(r, oracle_results(wl, range(wl.n_sims)), "costliest first")
     check_best(sim, wl, r)
     sim.close()
-    # one wave: the default order; a subset: its own
-    for kw, order in (({}, 0), ({"subset": list(range(0, wl.n_sims, 3)), "max_resident_warps": 64}, 1)):
+    # one wave: the default order; a subset: its own; eight waves: only the
+    # last trace (two waves of 32 warps) takes its alpha = 1 points first
+    for kw, order in (({}, 0), ({"subset": list(range(0, wl.n_sims, 3)), "max_resident_warps": 64}, 1),
+                      ({"max_resident_warps": 32}, 3)):
         s2 = gpu(wl, force_generic=generic, **kw)
         assert s2.info()["work_order"] == order
+        if order == 3:
+            assert_same(s2.results(), r, "last traces' alpha = 1 points first")
         s2.close()
 
 
