@@ -473,7 +473,8 @@ int costliest_first(const hx_grid* grid, int32_t n_traces, int64_t n_calls, int6
   order->clear();
   const int32_t P = grid->n_points;
   const int64_t n_sims = (int64_t)n_traces * P;
-  if (n_sims <= resident_warps) return 0;
+  // a list longer than 2^24 entries (128 MiB) is not worth its device memory
+  if (n_sims <= resident_warps || n_sims > (int64_t(1) << 24)) return 0;
   std::vector<int32_t> hot, cold;
   for (int32_t p = P - 1; p >= 0; --p)
     (grid->alpha_fp[p] == hx::kScale && grid->dispatch_policy[p] == HX_DISPATCH_WB ? hot : cold).push_back(p);
