@@ -21,6 +21,8 @@ key.
 Family `div`: the reward pass's division without its divergent early
 return; a warp barrier after each simulation's per-lane initial state.
 
+Family `cache`: the call-record loads with an L2 evict-last policy.
+
 Family `micro`: the event key formed with one shift and a mask; the
 simulation's beta, beta as a float and 1 - alpha, or its alpha, kept in
 registers instead of re-read from shared memory.
@@ -234,6 +236,46 @@ _SYNC_INIT = [("""    W->akey = nq > 0 ? (((uint64_t)a.arrival[qb] << 7) | kArri
     __syncwarp();  // every lane's initial instance state is read by the others
 """)]
 
+# Call-record loads (read-only in the simulation kernel) with an L2
+# evict-last policy, so that the alpha = 1 heaps streaming through L2 evict
+# them last.
+_LDG_LAST = """__device__ __forceinline__ int4 ldg_last4(const void* a) {
+  int4 v;
+  asm("{\\n .reg .b64 pol;\\n createpolicy.fractional.L2::evict_last.b64 pol, 1.0;\\n"
+      " ld.global.L2::cache_hint.v4.s32 {%0, %1, %2, %3}, [%4], pol;\\n}"
+      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(a));
+  return v;
+}
+__device__ __forceinline__ int2 ldg_last2(const void* a) {
+  int2 v;
+  asm("{\\n .reg .b64 pol;\\n createpolicy.fractional.L2::evict_last.b64 pol, 1.0;\\n"
+      " ld.global.L2::cache_hint.v2.s32 {%0, %1}, [%2], pol;\\n}"
+      : "=r"(v.x), "=r"(v.y) : "l"(a));
+  return v;
+}
+__device__ __forceinline__ int64_t ldg_last8(const void* a) {
+  int64_t v;
+  asm("{\\n .reg .b64 pol;\\n createpolicy.fractional.L2::evict_last.b64 pol, 1.0;\\n"
+      " ld.global.L2::cache_hint.s64 %0, [%1], pol;\\n}"
+      : "=l"(v) : "l"(a));
+  return v;
+}
+
+__device__ __forceinline__ bool ent_better("""
+_REC_L2LAST = [("""__device__ __forceinline__ bool ent_better(""", _LDG_LAST),
+               ("""  const int64_t dl = r->deadline;
+  const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);""",
+                """  const int64_t dl = ldg_last8(&r->deadline);
+  const int4 tail = ldg_last4(&r->tbar);"""),
+               ("""        const CallRec* r = rec + rid;
+        const int4 tail = *reinterpret_cast<const int4*>(&r->tbar);
+        const int64_t est_m = r->ev[c.inst_type[m]].x;""",
+                """        const CallRec* r = rec + rid;
+        const int4 tail = ldg_last4(&r->tbar);
+        const int64_t est_m = ldg_last2(&r->ev[c.inst_type[m]]).x;"""),
+               ("""        const int2 ev0 = r->ev[ty0], ev1 = r->ev[ty1];""",
+                """        const int2 ev0 = ldg_last2(&r->ev[ty0]), ev1 = ldg_last2(&r->ev[ty1]);""")]
+
 _INLINE_DIGEST = [("""__device__ __noinline__ void digest_flush(""", """__device__ __forceinline__ void digest_flush(""")]
 _INLINE_TOPK = [("""__device__ __noinline__ void topk_insert_warp(""", """__device__ __forceinline__ void topk_insert_warp(""")]
 
@@ -267,6 +309,8 @@ VARIANTS = {
     # on every lane rather than on the entry's lane and shuffled 1.006 (now in
     # the library), both 0.998, pend_smem 0.994
     "heap": {"sift_noshfl": (_SIFT_NOSHFL, [])},
+    # measured on 64 ceiling traces (library 3975 / 3980 ms): 0.965
+    "cache": {"rec_l2last": (_REC_L2LAST, [])},
     # measured on 64 ceiling traces (3 runs each, library 4127 / 4131 ms):
     # sync_init 0.997, div_uniform 0.998, both 0.997 -- within the run-to-run
     # spread; t_queue is now zeroed before the existing barrier instead
