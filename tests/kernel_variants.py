@@ -21,7 +21,8 @@ key.
 Family `div`: the reward pass's division without its divergent early
 return; a warp barrier after each simulation's per-lane initial state.
 
-Family `cache`: the call-record loads with an L2 evict-last policy.
+Family `cache`: the call-record loads with an L2 evict-last policy; the
+heap sift's deeper child loads not allocated in L1, or evicted from it first.
 
 Family `micro`: the event key formed with one shift and a mask; the
 simulation's beta, beta as a float and 1 - alpha, or its alpha, kept in
@@ -276,6 +277,33 @@ _REC_L2LAST = [("""__device__ __forceinline__ bool ent_better(""", _LDG_LAST),
                ("""        const int2 ev0 = r->ev[ty0], ev1 = r->ev[ty1];""",
                 """        const int2 ev0 = ldg_last2(&r->ev[ty0]), ev1 = ldg_last2(&r->ev[ty1]);""")]
 
+# The heap sift's child loads below the top two levels with an L1 policy:
+# not allocated in L1, or allocated to be evicted first (they are rarely
+# read again), so that the 28 KB L1 keeps the call records.
+def _sift_l1(policy):
+    return [("""    if (child < m) {
+      const HeapEnt e = h[child];
+      ck = e.key;
+      cr = e.rid;
+      cs = e.svc;
+    }""", """    if (child < m) {
+      HeapEnt e;
+      if (first >= 33) {
+        int4 v;
+        asm volatile("ld.global.L1::POLICY.v4.s32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(h + child) : "memory");
+        e.key = (long long)(((unsigned long long)(unsigned)v.y << 32) | (unsigned)v.x);
+        e.rid = v.z;
+        e.svc = v.w;
+      } else {
+        e = h[child];
+      }
+      ck = e.key;
+      cr = e.rid;
+      cs = e.svc;
+    }""".replace("POLICY", policy))]
+
+
 _INLINE_DIGEST = [("""__device__ __noinline__ void digest_flush(""", """__device__ __forceinline__ void digest_flush(""")]
 _INLINE_TOPK = [("""__device__ __noinline__ void topk_insert_warp(""", """__device__ __forceinline__ void topk_insert_warp(""")]
 
@@ -309,8 +337,11 @@ VARIANTS = {
     # on every lane rather than on the entry's lane and shuffled 1.006 (now in
     # the library), both 0.998, pend_smem 0.994
     "heap": {"sift_noshfl": (_SIFT_NOSHFL, [])},
-    # measured on 64 ceiling traces (library 3975 / 3980 ms): 0.965
-    "cache": {"rec_l2last": (_REC_L2LAST, [])},
+    # measured on 64 ceiling traces (library 3975 / 3980 ms): rec_l2last
+    # 0.965; again (library 3985 / 3976 ms) 0.969, sift_noalloc 0.996,
+    # sift_evict_first 0.997
+    "cache": {"rec_l2last": (_REC_L2LAST, []), "sift_noalloc": (_sift_l1("no_allocate"), []),
+              "sift_evict_first": (_sift_l1("evict_first"), [])},
     # measured on 64 ceiling traces (3 runs each, library 4127 / 4131 ms):
     # sync_init 0.997, div_uniform 0.998, both 0.997 -- within the run-to-run
     # spread; t_queue is now zeroed before the existing barrier instead
