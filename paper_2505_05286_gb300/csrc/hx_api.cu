@@ -5,12 +5,14 @@
 #include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstdio>
 #include <cstddef>
 #include <cstring>
 #include <mutex>
 #include <new>
 #include <string>
+#include <thread>
 #include <vector>
 
 #include "hx_device.cuh"
@@ -259,7 +261,11 @@ int validate_trace(const hx_trace* tr, int ti, const hx_cluster* c, int64_t min_
   if (!tr->call_base) return fail(HX_ERR_INVALID, where + "call_base is NULL");
   if (tr->call_base[0] != 0 || tr->call_base[tr->n_queries] != tr->n_calls)
     return fail(HX_ERR_INVALID, where + "call_base must run from 0 to n_calls");
-  int64_t horizon = 0;
+  // the time horizon: the last arrival plus every call's cost bound
+  // ceil(prompt * 10^6 / min_prefill) + max(out, out_est) * max_decode;
+  // summed here as sum(prompt) and sum(decode part), the sum of the ceilings
+  // lying within n_calls above the ceiling of the sum
+  int64_t tok_sum = 0, dec_sum = 0;
   for (int32_t i = 0; i < tr->n_queries; ++i) {
     if (tr->arrival_us[i] < 0 || (i > 0 && tr->arrival_us[i] < tr->arrival_us[i - 1]))
       return fail(HX_ERR_INVALID, where + "arrivals must be non-negative and sorted");
@@ -294,9 +300,13 @@ int validate_trace(const hx_trace* tr, int ti, const hx_cluster* c, int64_t min_
       const int64_t p = tr->prompt[j], o = tr->out[j], oe = tr->out_est[j];
       if (p < 1 || p > kTokMax || o < 0 || o > kTokMax || oe < 0 || oe > kTokMax)
         return fail(HX_ERR_INVALID, where + "token counts out of range");
-      const int64_t bound = (p * 1000000 + min_prefill - 1) / min_prefill + std::max(o, oe) * max_decode;
-      if (bound >= kCostMax) return fail(HX_ERR_INVALID, where + "a call's cost exceeds 2^28 us");
-      horizon += bound;
+      // ceil(p * 10^6 / min_prefill) + dec >= 2^28, decided without a division:
+      // ceil(x / d) >= m exactly when x > (m - 1) * d
+      const int64_t dec = std::max(o, oe) * max_decode;
+      if (dec >= kCostMax || p * 1000000 > (kCostMax - 1 - dec) * min_prefill)
+        return fail(HX_ERR_INVALID, where + "a call's cost exceeds 2^28 us");
+      tok_sum += p;
+      dec_sum += dec;
     }
   }
   // fault windows stretch attempts (slow-down or timeout) and delay the rest
@@ -305,9 +315,56 @@ int validate_trace(const hx_trace* tr, int ti, const hx_cluster* c, int64_t min_
     stretch = std::max(stretch, std::max<int64_t>(c->faults[f].slow_fp, c->timeout_mult_fp));
     last = std::max(last, c->faults[f].t1_us);
   }
+  const int64_t widen = 1 + (stretch + HX_SCALE - 1) / HX_SCALE, halve = c->n_faults > 0 ? 1 : 2;
+  const __int128 tok_us = (__int128)tok_sum * 1000000;
+  const int64_t lower = (int64_t)((tok_us + min_prefill - 1) / min_prefill) + dec_sum;
+  const int64_t upper = lower + tr->n_calls;
+  if (upper <= kHorizonMax && upper * widen / halve + last <= kHorizonMax) return HX_OK;
+  // near the limit: the exact sum of the per-call bounds decides
+  int64_t horizon = 0;
+  for (int32_t j = 0; j < tr->n_calls; ++j)
+    horizon += (tr->prompt[j] * int64_t(1000000) + min_prefill - 1) / min_prefill +
+               std::max<int64_t>(tr->out[j], tr->out_est[j]) * max_decode;
   if (horizon > kHorizonMax) return fail(HX_ERR_INVALID, where + "time horizon exceeds 2^39 us");
-  horizon = horizon * (1 + (stretch + HX_SCALE - 1) / HX_SCALE) / (c->n_faults > 0 ? 1 : 2) + last;
+  horizon = horizon * widen / halve + last;
   if (horizon > kHorizonMax) return fail(HX_ERR_INVALID, where + "time horizon exceeds 2^39 us");
+  return HX_OK;
+}
+
+// fn(t) for t = 0 .. n_traces - 1 on up to 16 host threads, one trace at a
+// time each, when the traces hold enough calls to pay for the threads.
+template <class F>
+void for_each_trace(const hx_trace* traces, int32_t n_traces, F fn) {
+  int64_t calls = 0;
+  for (int32_t t = 0; t < n_traces; ++t) calls += traces[t].n_calls;
+  const int64_t hw = std::max<int64_t>(1, std::thread::hardware_concurrency());
+  const int nt = (int)std::min<int64_t>({16, hw, (int64_t)n_traces, calls / 200000 + 1});
+  if (nt <= 1) {
+    for (int32_t t = 0; t < n_traces; ++t) fn(t);
+    return;
+  }
+  std::atomic<int32_t> next{0};
+  auto work = [&]() {
+    for (int32_t t; (t = next.fetch_add(1)) < n_traces;) fn(t);
+  };
+  std::vector<std::thread> pool;
+  for (int i = 1; i < nt; ++i) pool.emplace_back(work);
+  work();
+  for (std::thread& th : pool) th.join();
+}
+
+// validate_trace over every trace, in parallel; the lowest-numbered failing
+// trace's status and message are reported, as a loop in order would.
+int validate_traces(const hx_trace* traces, int32_t n_traces, const hx_cluster* c, int64_t min_prefill,
+                    int64_t max_decode) {
+  std::vector<int> rc((size_t)n_traces, HX_OK);
+  std::vector<std::string> msg((size_t)n_traces);
+  for_each_trace(traces, n_traces, [&](int32_t t) {
+    rc[t] = validate_trace(&traces[t], t, c, min_prefill, max_decode);
+    if (rc[t] != HX_OK) msg[t] = g_err;  // this thread's message
+  });
+  for (int32_t t = 0; t < n_traces; ++t)
+    if (rc[t] != HX_OK) return fail(rc[t], msg[t]);
   return HX_OK;
 }
 
@@ -335,18 +392,22 @@ std::vector<int32_t> tenant_kcaps(const hx_trace* traces, int32_t n_traces) {
 int upload_traces(hx_sim* h, const hx_trace* traces, cudaStream_t s) {
   std::vector<int64_t> arrival((size_t)h->n_q), qcall((size_t)h->n_q + 1);
   std::vector<uint8_t> kq((size_t)h->n_q), tenant((size_t)h->n_q, 0);
-  int64_t qo = 0, co = 0;
+  std::vector<int64_t> q0((size_t)h->n_traces + 1, 0), c0((size_t)h->n_traces + 1, 0);
   for (int t = 0; t < h->n_traces; ++t) {
+    q0[t + 1] = q0[t] + traces[t].n_queries;
+    c0[t + 1] = c0[t] + traces[t].n_calls;
+  }
+  for_each_trace(traces, h->n_traces, [&](int32_t t) {
     const hx_trace& tr = traces[t];
+    const int64_t qo = q0[t], co = c0[t];
     for (int32_t i = 0; i < tr.n_queries; ++i) {
       arrival[qo + i] = tr.arrival_us[i];
       kq[qo + i] = tr.k[i];
       qcall[qo + i] = co + tr.call_base[i];
       if (tr.tenant) tenant[qo + i] = tr.tenant[i];
     }
-    qo += tr.n_queries;
-    co += tr.n_calls;
-  }
+  });
+  int64_t co = c0[h->n_traces];
   qcall[h->n_q] = co;
   int rc;
   if ((rc = upload(h->d_arrival, arrival.data(), h->n_q, s)) || (rc = upload(h->d_k, kq.data(), h->n_q, s)) ||
@@ -511,8 +572,7 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   int rc;
   if ((rc = validate_cluster(cluster, &min_prefill, &max_decode))) return rc;
   if ((rc = validate_grid(grid))) return rc;
-  for (int t = 0; t < n_traces; ++t)
-    if ((rc = validate_trace(&traces[t], t, cluster, min_prefill, max_decode))) return rc;
+  if ((rc = validate_traces(traces, n_traces, cluster, min_prefill, max_decode))) return rc;
   if (opt && opt->n_record < 0) return fail(HX_ERR_INVALID, "n_record < 0");
   if (opt && opt->n_record > 0) {
     if (!opt->record_sims) return fail(HX_ERR_INVALID, "record_sims is NULL");
@@ -690,10 +750,8 @@ int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* str
   c.timeout_mult_fp = h->ck.timeout_mult_fp;
   c.n_faults = (int32_t)h->faults.size();
   c.faults = h->faults.data();
-  for (int t = 0; t < n_traces; ++t) {
-    int rc = validate_trace(&traces[t], t, &c, min_prefill, max_decode);
-    if (rc) return rc;
-  }
+  int rc = validate_traces(traces, n_traces, &c, min_prefill, max_decode);
+  if (rc) return rc;
   return upload_traces(h, traces, static_cast<cudaStream_t>(stream));
 }
 

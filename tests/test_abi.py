@@ -165,6 +165,43 @@ def test_rejects_malformed_inputs_without_device_work(lib):
         assert not h.value
 
 
+def test_parallel_validation_names_the_first_bad_trace(lib):
+    # about half a million calls: the traces are validated on several host
+    # threads, and the error still names the lowest-numbered bad trace
+    wl = W.make_workload(4, n_traces=8, n_queries=8000)
+    trs = [_copy_trace(t) for t in wl.traces]
+    trs[5].prompt[3] = 0
+    trs[2].arrival_us[4] = trs[2].arrival_us[3] - 1
+    trs[7].k[1] = 9
+    rc, err, h = _create(lib, trs, wl.cluster, wl.grid)
+    assert rc == H.HX_ERR_INVALID and err.startswith("trace 2:") and "sorted" in err, err
+    assert not h.value
+    trs[2] = _copy_trace(wl.traces[2])
+    rc, err, h = _create(lib, trs, wl.cluster, wl.grid)
+    assert rc == H.HX_ERR_INVALID and err.startswith("trace 5:") and "token" in err, err
+
+
+def test_horizon_limit_is_exact(lib):
+    # without fault windows the horizon is the sum over calls of
+    # ceil(prompt * 10^6 / min prefill rate) + max(out, out_est) * max decode
+    # time, plus the last arrival; 2^39 us is allowed, one more is not
+    wl = W.make_workload(0, n_queries=20)
+    c, tr = wl.cluster, wl.traces[0]
+    mp, md = int(np.min(c.prefill_tok_s)), int(np.max(c.decode_us_tok))
+    hz = sum(-(-int(p) * 10 ** 6 // mp) + max(int(o), int(oe)) * md
+             for p, o, oe in zip(tr.prompt, tr.out, tr.out_est))
+    for extra, accepted in ((0, True), (1, False)):
+        t = _copy_trace(tr)
+        t.arrival_us += (1 << 39) - hz - int(tr.arrival_us[-1]) + extra
+        rc, err, h = _create(lib, [t], c, wl.grid)
+        if accepted:
+            assert rc != H.HX_ERR_INVALID, err  # validation passed (HX_ERR_CUDA without a GPU)
+            if h.value:
+                lib.hx_sim_destroy(h)
+        else:
+            assert rc == H.HX_ERR_INVALID and "horizon" in err, err
+
+
 def test_rejects_bad_options(lib):
     wl = W.make_workload(0, n_queries=20)  # 1 trace x 16 points
 
