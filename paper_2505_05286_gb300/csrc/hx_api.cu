@@ -9,7 +9,11 @@
 #include <cstdio>
 #include <cstddef>
 #include <cstring>
+#include <exception>
+#include <memory>
 #include <mutex>
+#include <stdexcept>
+#include <system_error>
 #include <new>
 #include <string>
 #include <thread>
@@ -32,6 +36,29 @@ struct NvtxRange {
 
 int fail(int code, const std::string& msg) {
   g_err = msg;
+  return code;
+}
+
+// Host-side C++ exceptions (an allocation that fails) become a status
+// here instead of crossing the C ABI.
+template <class F>
+int guarded(F&& f) noexcept {
+  const char* msg = "unexpected host exception";
+  int code = HX_ERR_STATE;
+  try {
+    return f();
+  } catch (const std::bad_alloc&) {
+    msg = "host allocation failed";
+    code = HX_ERR_OOM;
+  } catch (const std::length_error&) {
+    msg = "host allocation failed";
+    code = HX_ERR_OOM;
+  } catch (...) {
+  }
+  try {
+    g_err = msg;
+  } catch (...) {
+  }
   return code;
 }
 
@@ -344,13 +371,26 @@ void for_each_trace(const hx_trace* traces, int32_t n_traces, F fn) {
     return;
   }
   std::atomic<int32_t> next{0};
+  std::mutex m;
+  std::exception_ptr first;  // the first exception a worker met, thrown again below
   auto work = [&]() {
-    for (int32_t t; (t = next.fetch_add(1)) < n_traces;) fn(t);
+    try {
+      for (int32_t t; (t = next.fetch_add(1)) < n_traces;) fn(t);
+    } catch (...) {
+      std::lock_guard<std::mutex> lock(m);
+      if (!first) first = std::current_exception();
+      next = n_traces;  // the others stop at their next trace
+    }
   };
   std::vector<std::thread> pool;
-  for (int i = 1; i < nt; ++i) pool.emplace_back(work);
+  try {
+    for (int i = 1; i < nt; ++i) pool.emplace_back(work);
+  } catch (const std::system_error&) {
+    // fewer threads than asked for: those started and this one share the traces
+  }
   work();
   for (std::thread& th : pool) th.join();
+  if (first) std::rethrow_exception(first);
 }
 
 // validate_trace over every trace, in parallel; the lowest-numbered failing
@@ -561,8 +601,8 @@ extern "C" {
 
 const char* hx_last_error(void) { return g_err.c_str(); }
 
-int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cluster, const hx_grid* grid,
-                  const hx_options* opt, hx_sim** out) {
+static int hx_sim_create_impl(const hx_trace* traces, int32_t n_traces, const hx_cluster* cluster, const hx_grid* grid,
+                              const hx_options* opt, hx_sim** out) {
   NvtxRange range("hx_sim_create");
   if (!out) return fail(HX_ERR_INVALID, "out is NULL");
   *out = nullptr;
@@ -588,12 +628,11 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
   std::vector<int64_t> subset;
   if ((rc = order_subset(opt, n_traces, grid->n_points, &subset))) return rc;
 
-  hx_sim* h = new (std::nothrow) hx_sim();
+  // the handle is freed on every early return (and exception) until it is handed out
+  std::unique_ptr<hx_sim> owner(new (std::nothrow) hx_sim());
+  hx_sim* h = owner.get();
   if (!h) return fail(HX_ERR_OOM, "host allocation failed");
-  auto bail = [&](int code) {
-    delete h;
-    return code;
-  };
+  auto bail = [](int code) { return code; };
   h->n_traces = n_traces;
   h->n_points = grid->n_points;
   h->n_sims = (int64_t)n_traces * grid->n_points;
@@ -726,11 +765,11 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
       if (cudaEventCreate(&e) != cudaSuccess) return bail(fail(HX_ERR_CUDA, "cudaEventCreate failed"));
   }
   if (cudaDeviceSynchronize() != cudaSuccess) return bail(fail(HX_ERR_CUDA, "upload failed"));
-  *out = h;
+  *out = owner.release();
   return HX_OK;
 }
 
-int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream) {
+static int hx_sim_upload_impl(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream) {
   NvtxRange range("hx_sim_upload");
   if (!h || !traces) return fail(HX_ERR_INVALID, "NULL argument");
   if (n_traces != h->n_traces) return fail(HX_ERR_INVALID, "trace count differs from the handle's");
@@ -755,7 +794,7 @@ int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* str
   return upload_traces(h, traces, static_cast<cudaStream_t>(stream));
 }
 
-int hx_sim_run(hx_sim* h, void* stream) {
+static int hx_sim_run_impl(hx_sim* h, void* stream) {
   NvtxRange range("hx_sim_run");
   if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -848,7 +887,7 @@ int hx_sim_run(hx_sim* h, void* stream) {
   return HX_OK;
 }
 
-int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n) {
+static int hx_sim_results_impl(hx_sim* h, hx_result* host_out, size_t n) {
   NvtxRange range("hx_sim_results");
   if (!h || !host_out) return fail(HX_ERR_INVALID, "NULL argument");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
@@ -858,7 +897,7 @@ int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n) {
   return HX_OK;
 }
 
-int hx_sim_extras(hx_sim* h, hx_extra* host_out, size_t n) {
+static int hx_sim_extras_impl(hx_sim* h, hx_extra* host_out, size_t n) {
   if (!h || !host_out) return fail(HX_ERR_INVALID, "NULL argument");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
   if ((int64_t)n > h->n_sims) return fail(HX_ERR_INVALID, "n exceeds the number of simulations");
@@ -881,7 +920,7 @@ int hx_sim_extras(hx_sim* h, hx_extra* host_out, size_t n) {
   return HX_OK;
 }
 
-int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out) {
+static int hx_sim_best_impl(hx_sim* h, int32_t objective, hx_best* out) {
   if (!h || !out) return fail(HX_ERR_INVALID, "NULL argument");
   if (objective != HX_OBJ_P95 && objective != HX_OBJ_P95_SLO95) return fail(HX_ERR_INVALID, "unknown objective");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
@@ -904,7 +943,8 @@ int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out) {
   return HX_OK;
 }
 
-int hx_sim_point_sums(hx_sim* h, int64_t* sum_p95, int64_t* sum_slo_met, int32_t* n_failed, size_t n_points) {
+static int hx_sim_point_sums_impl(hx_sim* h, int64_t* sum_p95, int64_t* sum_slo_met, int32_t* n_failed,
+                                  size_t n_points) {
   if (!h || !sum_p95 || !sum_slo_met || !n_failed) return fail(HX_ERR_INVALID, "NULL argument");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
   if ((int64_t)n_points != h->n_points) return fail(HX_ERR_INVALID, "n_points differs from the handle's");
@@ -919,8 +959,8 @@ int hx_sim_point_sums(hx_sim* h, int64_t* sum_p95, int64_t* sum_slo_met, int32_t
   return HX_OK;
 }
 
-int hx_best_of_sums(const int64_t* sum_p95, const int64_t* sum_slo_met, const int32_t* n_failed, int32_t n_points,
-                    int64_t n_queries_total, int32_t objective, hx_best* out) {
+static int hx_best_of_sums_impl(const int64_t* sum_p95, const int64_t* sum_slo_met, const int32_t* n_failed,
+                                int32_t n_points, int64_t n_queries_total, int32_t objective, hx_best* out) {
   if (!sum_p95 || !sum_slo_met || !n_failed || !out) return fail(HX_ERR_INVALID, "NULL argument");
   if (n_points < 1 || n_queries_total < 0) return fail(HX_ERR_INVALID, "bad sizes");
   if (objective != HX_OBJ_P95 && objective != HX_OBJ_P95_SLO95) return fail(HX_ERR_INVALID, "unknown objective");
@@ -969,8 +1009,8 @@ int hx_best_of_sums(const int64_t* sum_p95, const int64_t* sum_slo_met, const in
   return rc;
 }
 
-int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us, int64_t* budget_us,
-                   int64_t* start_us, int64_t* end_us, size_t n_calls) {
+static int hx_sim_records_impl(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us, int64_t* budget_us,
+                               int64_t* start_us, int64_t* end_us, size_t n_calls) {
   if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
   if (rec_index < 0 || rec_index >= h->n_record) return fail(HX_ERR_INVALID, "rec_index out of range");
@@ -987,8 +1027,8 @@ int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us,
   return HX_OK;
 }
 
-int hx_sim_prep(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int32_t* tbar, int64_t* deadline_us,
-                size_t n_calls) {
+static int hx_sim_prep_impl(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int32_t* tbar,
+                            int64_t* deadline_us, size_t n_calls) {
   if (!h) return fail(HX_ERR_INVALID, "handle is NULL");
   if (!h->ran) return fail(HX_ERR_STATE, "hx_sim_run has not been called");
   if (trace_index < 0 || trace_index >= h->n_traces) return fail(HX_ERR_INVALID, "trace_index out of range");
@@ -1142,8 +1182,8 @@ struct Carve {
 
 }  // namespace
 
-extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluster, const hx_grid* grid,
-                                 int32_t objective, hx_result* results, hx_best* best, void* stream) {
+static int hx_sim_run_static_impl(const hx_trace* trace, const hx_cluster* cluster, const hx_grid* grid,
+                                  int32_t objective, hx_result* results, hx_best* best, void* stream) {
   g_err.clear();
   if (!trace || !results) return fail(HX_ERR_INVALID, "trace and results must not be NULL");
   if (objective != HX_OBJ_P95 && objective != HX_OBJ_P95_SLO95) return fail(HX_ERR_INVALID, "unknown objective");
@@ -1317,3 +1357,60 @@ extern "C" int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluste
   }
   return HX_OK;
 }
+
+// The C entry points: each runs its implementation above under guarded(), so
+// that no C++ exception crosses the ABI.
+extern "C" {
+
+int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cluster, const hx_grid* grid,
+                  const hx_options* opt, hx_sim** out) {
+  return guarded([&] { return hx_sim_create_impl(traces, n_traces, cluster, grid, opt, out); });
+}
+
+int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream) {
+  return guarded([&] { return hx_sim_upload_impl(h, traces, n_traces, stream); });
+}
+
+int hx_sim_run(hx_sim* h, void* stream) {
+  return guarded([&] { return hx_sim_run_impl(h, stream); });
+}
+
+int hx_sim_results(hx_sim* h, hx_result* host_out, size_t n) {
+  return guarded([&] { return hx_sim_results_impl(h, host_out, n); });
+}
+
+int hx_sim_extras(hx_sim* h, hx_extra* host_out, size_t n) {
+  return guarded([&] { return hx_sim_extras_impl(h, host_out, n); });
+}
+
+int hx_sim_best(hx_sim* h, int32_t objective, hx_best* out) {
+  return guarded([&] { return hx_sim_best_impl(h, objective, out); });
+}
+
+int hx_sim_point_sums(hx_sim* h, int64_t* sum_p95, int64_t* sum_slo_met, int32_t* n_failed, size_t n_points) {
+  return guarded([&] { return hx_sim_point_sums_impl(h, sum_p95, sum_slo_met, n_failed, n_points); });
+}
+
+int hx_best_of_sums(const int64_t* sum_p95, const int64_t* sum_slo_met, const int32_t* n_failed, int32_t n_points,
+                    int64_t n_queries_total, int32_t objective, hx_best* out) {
+  return guarded(
+      [&] { return hx_best_of_sums_impl(sum_p95, sum_slo_met, n_failed, n_points, n_queries_total, objective, out); });
+}
+
+int hx_sim_records(hx_sim* h, int32_t rec_index, int32_t* inst, int64_t* enq_us, int64_t* budget_us,
+                   int64_t* start_us, int64_t* end_us, size_t n_calls) {
+  return guarded(
+      [&] { return hx_sim_records_impl(h, rec_index, inst, enq_us, budget_us, start_us, end_us, n_calls); });
+}
+
+int hx_sim_prep(hx_sim* h, int32_t trace_index, int32_t* est, int32_t* svc, int32_t* tbar, int64_t* deadline_us,
+                size_t n_calls) {
+  return guarded([&] { return hx_sim_prep_impl(h, trace_index, est, svc, tbar, deadline_us, n_calls); });
+}
+
+int hx_sim_run_static(const hx_trace* trace, const hx_cluster* cluster, const hx_grid* grid,
+                      int32_t objective, hx_result* results, hx_best* best, void* stream) {
+  return guarded([&] { return hx_sim_run_static_impl(trace, cluster, grid, objective, results, best, stream); });
+}
+
+}  // extern "C"
