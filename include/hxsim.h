@@ -237,8 +237,11 @@ int hx_sim_create(const hx_trace* traces, int32_t n_traces, const hx_cluster* cl
 
 /* Replace the trace contents of an existing handle with traces of the same
  * shapes (n_queries and n_calls per trace), copying host -> device on
- * `stream`; no allocation.  A trace whose tenant pointer is NULL puts every
- * query in tenant 0, as at create. */
+ * `stream`; no device allocation.  The traces are validated as at create
+ * (on up to 16 host threads; the lowest-numbered bad trace is reported)
+ * before anything is copied, and the call returns once the copies are done.
+ * A trace whose tenant pointer is NULL puts every query in tenant 0, as at
+ * create.  Errors: HX_ERR_INVALID, HX_ERR_OOM (host staging), HX_ERR_CUDA. */
 int hx_sim_upload(hx_sim* h, const hx_trace* traces, int32_t n_traces, void* stream);
 
 /* Enqueue the whole path on `stream` (a cudaStream_t, NULL = legacy default):
