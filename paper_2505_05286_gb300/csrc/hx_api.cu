@@ -383,10 +383,13 @@ void for_each_trace(const hx_trace* traces, int32_t n_traces, F fn) {
     }
   };
   std::vector<std::thread> pool;
-  try {
-    for (int i = 1; i < nt; ++i) pool.emplace_back(work);
-  } catch (const std::system_error&) {
-    // fewer threads than asked for: those started and this one share the traces
+  pool.reserve((size_t)nt - 1);  // any allocation failure comes before a thread starts
+  for (int i = 1; i < nt; ++i) {
+    try {
+      pool.emplace_back(work);
+    } catch (const std::system_error&) {
+      break;  // fewer threads than asked for: those started and this one share the traces
+    }
   }
   work();
   for (std::thread& th : pool) th.join();
